@@ -1,0 +1,95 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each case plants one mistake in a copy of the oracle's source (on the CPU,
+never in the CUDA path) and checks that at least one pin then fails: the
+hand-derived closed forms of tests/golden or the brute force.
+"""
+import inspect
+import json
+import os
+import types
+
+import numpy as np
+import pytest
+
+from oracle import timebill_oracle as orc
+from tests import brute_force as bf
+from tests.test_oracle_pins import GOLDEN, _frac_expr, _golden_vote_inputs
+
+SRC = inspect.getsource(orc)
+
+MUTANTS = {
+    "scale 1/d instead of 1/sqrt(d)": ("sigma = 1.0 / math.sqrt(d)\n    # visible", "sigma = 1.0 / d\n    # visible"),
+    "window row sees one key too few": ("<= (P + np.arange(W))", "< (P + np.arange(W))"),
+    "window row sees the whole window": ("<= (P + np.arange(W))[:, None]", "<= (P + W - 1 + 0 * np.arange(W))[:, None]"),
+    "window keys also scored": ("S[g] += prob[:, :P].sum(axis=0)", "S[g] += prob[:, 1:P + 1].sum(axis=0)"),
+    "interleaved head mapping": ("for h in range(g * G, (g + 1) * G):\n            logits", "for h in range(g, hq, hkv):\n            logits"),
+    "pool misses right neighbours": ("out[..., :-t] = np.maximum(out[..., :-t], S[..., t:])", "pass"),
+    "pool one wider": ("range(1, pool_k // 2 + 1)", "range(1, pool_k // 2 + 2)"),
+    "ties to the higher index": ("np.lexsort((np.arange(P), -pooled))", "np.lexsort((-np.arange(P), -pooled))"),
+    "budget rounds instead of ceil": ("k = math.ceil((1.0 - alpha) * n - 1e-9 * n)", "k = round((1.0 - alpha) * n)"),
+    "budget counts the window inside": ("return k, k + window", "return max(k - window, 0), max(k - window, 0) + window"),
+    "decode scale dropped": ("s = sigma * (kk @ q[h])", "s = kk @ q[h]"),
+    "decode attends one row too many": ("kk = np.asarray(Kc[g, :length]", "kk = np.asarray(Kc[g, :length + 1]"),
+}
+
+
+def _mutant(name):
+    old, new = MUTANTS[name]
+    assert SRC.count(old) == 1, name
+    mod = types.ModuleType("oracle_mutant")
+    exec(compile(SRC.replace(old, new), "oracle_mutant", "exec"), mod.__dict__)
+    return mod
+
+
+def _pins_pass(m):
+    """Run a compact version of the pins against module m; False on any miss."""
+    try:
+        with open(os.path.join(GOLDEN, "window_vote_closed_form.json")) as f:
+            gd = json.load(f)
+        q, K = _golden_vote_inputs(gd)
+        if m.retained_count(6, 2, gd["alpha"]) != (2, 4):
+            return False
+        if m.retained_count(131072, 64, 0.9) != (13108, 13172):
+            return False
+        S = m.window_scores(q, K)
+        S_exp = np.array([[_frac_expr(x) for x in r] for r in gd["S_expected"]])
+        if not np.allclose(S, S_exp, rtol=1e-12, atol=0):
+            return False
+        for case in gd["cases"]:
+            pooled = m.max_pool(S, case["pool_k"])
+            for g in range(2):
+                if m.select_indices(pooled[g], 2, 6).tolist() != case["idx_expected"][g]:
+                    return False
+        rng = np.random.default_rng(2)
+        qq = rng.standard_normal((3, 5, 8))
+        KK = rng.standard_normal((1, 33, 8)) * 1.5
+        VV = rng.standard_normal((1, 33, 8))
+        S2 = m.window_scores(qq, KK)
+        S2_bf = np.array(bf.scores(qq.tolist(), KK.tolist(), 3))
+        if not np.allclose(S2, S2_bf, rtol=1e-12):
+            return False
+        pb = bf.pool(S2_bf[0].tolist(), 7)
+        if not np.allclose(m.max_pool(S2, 7)[0], pb, rtol=1e-12):
+            return False
+        # exact ties: constant keys
+        Kt = np.tile(KK[:, :1], (1, 33, 1))
+        pt = m.max_pool(m.window_scores(qq, Kt), 7)[0]
+        if m.select_indices(pt, 10, 33).tolist() != bf.select(pt.tolist(), 10, 33):
+            return False
+        out = m.decode_attention(qq[:1, 0], KK, VV, 20)
+        ref = bf.attention(qq[0, 0].tolist(), KK[0].tolist(), VV[0].tolist(), 20)
+        if not np.allclose(out[0], ref, rtol=1e-12):
+            return False
+        return True
+    except (ValueError, IndexError, AssertionError):
+        return False
+
+
+def test_unmutated_oracle_passes():
+    assert _pins_pass(orc)
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name):
+    assert not _pins_pass(_mutant(name)), name
