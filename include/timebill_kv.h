@@ -1,0 +1,217 @@
+/*
+ * timebill_kv.h - C ABI of the GB300 (sm_103a) KV-eviction + decode-attention
+ * library behind TimeBill's eviction ratio alpha (arxiv 2512.21859).
+ *
+ * The paper chooses, per request, the fraction alpha of the prompt's KV cache
+ * to evict after prefill (Eq. 14, Section "Time-Budgeted LLM Inference
+ * Mechanism"), so that every decode step then attends over
+ * N_kv = (1 - alpha) N_x + i - 1 keys (Eq. 8, Section "End-to-end Execution
+ * Time Prediction"). It performs the eviction with SnapKV ("Experimental
+ * Setup"). This library computes that eviction and the decode-step
+ * attention over the compacted cache; choosing alpha stays with the caller.
+ *
+ * Conventions shared by every entry point
+ * ----------------------------------------
+ *  - The caller owns every buffer. Device buffers hold device addresses
+ *    (allocated by the caller, e.g. with PyTorch); descriptor arrays marked
+ *    "host" hold host addresses read during the call only. The library never
+ *    allocates device memory; scratch comes from a caller-provided workspace
+ *    whose size the *_workspace_size functions report.
+ *  - Device calls are asynchronous on the given stream (NULL = the legacy
+ *    default stream). Argument errors are returned synchronously, before
+ *    anything is launched; the output buffers are then left untouched.
+ *  - bf16 tensors are raw 16-bit bfloat16 values; f32 tensors IEEE float.
+ *    Every device pointer must be 16-byte aligned.
+ *  - No exceptions cross the ABI; every call returns a tb_status.
+ *  - Calls that share a workspace must not overlap on the GPU.
+ *
+ * Notation: B requests; request b has prompt length N_b, eviction ratio
+ * alpha_b and P_b = N_b - W prefix tokens (the last W prompt tokens form the
+ * observation window). Hq query heads, Hkv KV heads, G = Hq / Hkv; query head
+ * h reads KV head h / G. d = head_dim. k_b retained prefix tokens and
+ * R_b = k_b + W retained rows per KV head (tb_retained_count).
+ *
+ * Packed layouts (row-major, innermost index last):
+ *   q_win   [B][Hq][W][d]           window queries (the last W prompt rows)
+ *   K, V    [Hkv][kv_rows][d]       request b at rows kv_offset[b] .. + N_b
+ *   scores  [Hkv][score_rows] f32   request b at column sum_{b'<b} P_b'
+ *   idx     [Hkv][idx_rows] int32   request b at column sum_{b'<b} R_b'
+ *   Kc, Vc  [Hkv][out_rows][d]      request b at rows out_offset[b] .. + R_b
+ *   score_rows = sum_b P_b, idx_rows = sum_b R_b (see tb_evict_layout).
+ */
+#ifndef TIMEBILL_KV_H
+#define TIMEBILL_KV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream (cudaStream_t). */
+typedef struct CUstream_st *tb_stream_t;
+
+typedef enum {
+  TB_OK = 0,
+  TB_ERR_INVALID_ARG = 1,  /* null pointer, bad size, inconsistent layout */
+  TB_ERR_UNSUPPORTED = 2,  /* valid but not built: head_dim, dtype, batch */
+  TB_ERR_WORKSPACE = 3,    /* workspace missing, too small or misaligned */
+  TB_ERR_CUDA = 4,         /* a CUDA launch or runtime call failed */
+  TB_ERR_TIMEOUT = 5       /* a bounded device-side wait gave up */
+} tb_status;
+
+typedef enum { TB_F32 = 0, TB_BF16 = 1 } tb_dtype;
+
+/* Largest batch one call accepts. */
+#define TB_MAX_BATCH 64
+
+/* Static description of a status code; never NULL. */
+const char *tb_status_string(int32_t status);
+
+/* Version of this ABI (major * 100 + minor). */
+int32_t tb_abi_version(void);
+
+/* Text of the last CUDA error this thread saw inside the library (the
+ * cudaGetErrorString of the call behind a TB_ERR_CUDA), or "" if none. */
+const char *tb_last_error_detail(void);
+
+/* Kernels this library has launched in this process so far (all threads,
+ * all devices). Lets a caller count the device work behind a region. */
+uint64_t tb_launch_counter(void);
+
+/*
+ * Retained length (Eq. 8). k = ceil((1 - alpha) n - 1e-9 n) prefix tokens
+ * survive on top of the W window tokens, clamped to [0, n - window]; the
+ * 1e-9 n guard keeps a decimal alpha (0.3) from rounding up past an exact
+ * product. Writes k to *k_out and k + window to *r_out.
+ * Errors: TB_ERR_INVALID_ARG if a pointer is NULL, window < 1, n < window,
+ * or alpha is outside [0, 1] (NaN included).
+ */
+tb_status tb_retained_count(int64_t n, int32_t window, double alpha,
+                            int64_t *k_out, int64_t *r_out);
+
+/* Shape of one batched eviction. All pointers are host arrays of length
+ * `batch`, read during the call only. */
+typedef struct {
+  int32_t batch;     /* 1 .. TB_MAX_BATCH */
+  int32_t hq;        /* query heads, a multiple of hkv */
+  int32_t hkv;       /* KV heads */
+  int32_t head_dim;  /* 64 or 128 */
+  int32_t window;    /* observation window W >= 1 (W <= N_b) */
+  int32_t pool_k;    /* max-pool kernel, odd, 1 .. 63 */
+  int32_t dtype;     /* tb_dtype of q_win, K, V, Kc, Vc */
+  int32_t reserved;  /* must be 0 */
+  const int64_t *n;          /* host [batch]: prompt lengths N_b */
+  const double *alpha;       /* host [batch]: eviction ratios in [0, 1] */
+  const int64_t *kv_offset;  /* host [batch]: first row of request b in K, V */
+  int64_t kv_rows;           /* rows per KV head of K and V */
+  const int64_t *out_offset; /* host [batch]: first row of request b in Kc, Vc */
+  const int64_t *out_cap;    /* host [batch]: rows reserved for b (>= R_b) */
+  int64_t out_rows;          /* rows per KV head of Kc and Vc */
+} tb_evict_desc;
+
+/*
+ * Validates a descriptor and reports the packed sizes: *score_rows =
+ * sum_b P_b and *idx_rows = sum_b R_b (either pointer may be NULL).
+ * Errors: TB_ERR_INVALID_ARG (inconsistent descriptor, request rows outside
+ * kv_rows / out_rows, out_cap < R_b), TB_ERR_UNSUPPORTED (head_dim, dtype).
+ */
+tb_status tb_evict_layout(const tb_evict_desc *desc, int64_t *score_rows,
+                          int64_t *idx_rows);
+
+/* Bytes of device workspace tb_window_scores, tb_select_topk and
+ * tb_score_evict need for this descriptor (the same figure for all three). */
+tb_status tb_evict_workspace_size(const tb_evict_desc *desc, size_t *bytes);
+
+/*
+ * Steps 1-3 of the eviction (SnapKV observation-window voting, named in
+ * "Experimental Setup"; logits and softmax of the attention definition in
+ * "FLOPs-based Modeling"): for every request, KV head g and prefix key j,
+ *   scores[g][j] = sum over heads h of group g and window rows w of
+ *                  softmax_j'( q_win[h][w] . K[g][j'] / sqrt(d) )[j],
+ * where window row w sees keys j' <= P_b + w (causal). Writes `scores`
+ * ([Hkv][score_rows] f32, device). Reads q_win, K (device).
+ */
+tb_status tb_window_scores(const tb_evict_desc *desc, const void *q_win,
+                           const void *K, float *scores, void *workspace,
+                           size_t workspace_bytes, tb_stream_t stream);
+
+/*
+ * Steps 4-5: max-pool of the scores (kernel pool_k, stride 1, out-of-range
+ * neighbours ignored), then per request and KV head the k_b prefix positions
+ * with the largest pooled score (ties to the lower index) followed by the
+ * window positions P_b .. N_b - 1, ascending, into idx ([Hkv][idx_rows]
+ * int32, device; positions are relative to the request's first row).
+ * `pooled` ([Hkv][score_rows] f32, device) receives the pooled scores, or
+ * is NULL. Scores must be finite and >= 0.
+ */
+tb_status tb_select_topk(const tb_evict_desc *desc, const float *scores,
+                         int32_t *idx, float *pooled, void *workspace,
+                         size_t workspace_bytes, tb_stream_t stream);
+
+/*
+ * Step 6: Kc[g][out_offset[b] + r] = K[g][kv_offset[b] + idx[g][.. + r]]
+ * and the same for V, for r < R_b (bit copies). idx entries must lie in
+ * [0, N_b); an entry outside it is skipped and its row left untouched.
+ */
+tb_status tb_gather_kv(const tb_evict_desc *desc, const int32_t *idx,
+                       const void *K, const void *V, void *Kc, void *Vc,
+                       tb_stream_t stream);
+
+/*
+ * The whole eviction: tb_window_scores, tb_select_topk and tb_gather_kv in
+ * one call (scores kept in the workspace). `pooled` may be NULL.
+ */
+tb_status tb_score_evict(const tb_evict_desc *desc, const void *q_win,
+                         const void *K, const void *V, int32_t *idx,
+                         void *Kc, void *Vc, float *pooled, void *workspace,
+                         size_t workspace_bytes, tb_stream_t stream);
+
+/* Shape of one batched decode step. */
+typedef struct {
+  int32_t batch;     /* 1 .. TB_MAX_BATCH */
+  int32_t hq;        /* query heads, a multiple of hkv */
+  int32_t hkv;       /* KV heads */
+  int32_t head_dim;  /* 64 or 128 */
+  int32_t dtype;     /* tb_dtype of q, Kc, Vc */
+  int32_t out_dtype; /* tb_dtype of out: TB_F32, or equal to dtype */
+  const int64_t *cache_offset; /* host [batch]: first row of b in Kc, Vc */
+  const int64_t *cache_cap;    /* host [batch]: rows reserved for b */
+  int64_t cache_rows;          /* rows per KV head of Kc and Vc */
+  int64_t max_len;             /* upper bound of lens[b], >= 1 */
+} tb_decode_desc;
+
+/* Bytes of device workspace tb_decode_attn needs for this descriptor. */
+tb_status tb_decode_workspace_size(const tb_decode_desc *desc, size_t *bytes);
+
+/*
+ * One decode step (attention definition of "FLOPs-based Modeling" with a
+ * single query row; N_kv^i keys per Eq. 8): for request b and query head h,
+ *   out[b][h] = sum_{r < lens[b]} softmax_r(q[b][h] . Kc[g][r] / sqrt(d)) Vc[g][r]
+ * with g = h / G and rows taken from request b's slice of Kc, Vc. The caller
+ * appends the step's own K/V row at lens[b] - 1 beforehand.
+ * q: [B][Hq][d] (dtype); out: [B][Hq][d] (out_dtype); lens: device int32 [B].
+ * A length above min(max_len, cache_cap[b]) is clamped to it and flagged in
+ * the workspace status word (tb_read_status); lens[b] <= 0 writes zeros.
+ */
+tb_status tb_decode_attn(const tb_decode_desc *desc, const void *q,
+                         const void *Kc, const void *Vc, const int32_t *lens,
+                         void *out, void *workspace, size_t workspace_bytes,
+                         tb_stream_t stream);
+
+/*
+ * Waits for `stream`, then reads the status word kept at the start of a
+ * workspace used by the calls above: TB_OK, TB_ERR_TIMEOUT (a bounded
+ * device-side wait gave up) or TB_ERR_INVALID_ARG (a device-side range check
+ * fired, e.g. a decode length above its cap). *raw (if not NULL) receives the
+ * word itself. The word is cleared at the start of every call.
+ */
+tb_status tb_read_status(const void *workspace, size_t workspace_bytes,
+                         tb_stream_t stream, int32_t *raw);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TIMEBILL_KV_H */

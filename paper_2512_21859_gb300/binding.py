@@ -1,0 +1,303 @@
+"""Thin ctypes binding of libtimebill_kv.so (C ABI: include/timebill_kv.h).
+
+Argument marshalling only: the functions below carry the C entry points'
+names, turn tensors into device pointers and host lists into the
+descriptor structs, and raise ``TbError`` on a non-OK status. Every step of
+the computation runs in the library's CUDA kernels. Device buffers may be
+torch tensors (their data_ptr() is passed) or plain integer addresses.
+If the library has not been built, the first call raises RuntimeError.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import numpy as np
+
+__all__ = [
+    "TB_OK", "TB_ERR_INVALID_ARG", "TB_ERR_UNSUPPORTED", "TB_ERR_WORKSPACE",
+    "TB_ERR_CUDA", "TB_ERR_TIMEOUT", "TB_F32", "TB_BF16", "TB_MAX_BATCH",
+    "TbError", "EvictDesc", "DecodeDesc", "library_path", "load",
+    "tb_status_string", "tb_abi_version", "tb_last_error_detail", "tb_launch_counter",
+    "tb_retained_count", "tb_evict_layout", "tb_evict_workspace_size",
+    "tb_window_scores", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
+    "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
+]
+
+TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
+TB_F32, TB_BF16 = 0, 1
+TB_MAX_BATCH = 64
+
+_I64P = ctypes.POINTER(ctypes.c_int64)
+_F64P = ctypes.POINTER(ctypes.c_double)
+
+
+class _EvictDescC(ctypes.Structure):
+    _fields_ = [
+        ("batch", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32), ("window", ctypes.c_int32), ("pool_k", ctypes.c_int32),
+        ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("n", _I64P), ("alpha", _F64P), ("kv_offset", _I64P), ("kv_rows", ctypes.c_int64),
+        ("out_offset", _I64P), ("out_cap", _I64P), ("out_rows", ctypes.c_int64),
+    ]
+
+
+class _DecodeDescC(ctypes.Structure):
+    _fields_ = [
+        ("batch", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32), ("dtype", ctypes.c_int32), ("out_dtype", ctypes.c_int32),
+        ("cache_offset", _I64P), ("cache_cap", _I64P), ("cache_rows", ctypes.c_int64),
+        ("max_len", ctypes.c_int64),
+    ]
+
+
+class TbError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        detail = ""
+        if status == TB_ERR_CUDA:
+            try:
+                detail = ": " + tb_last_error_detail()
+            except Exception:  # pragma: no cover
+                pass
+        super().__init__("%s failed: %s (status %d)%s" % (where, tb_status_string(status), status, detail))
+
+
+def library_path() -> str:
+    return os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtimebill_kv.so")
+
+
+_LIB = None
+
+
+def load():
+    """Loads the shared library (once) and declares the entry points."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = library_path()
+    if not os.path.exists(path):
+        raise RuntimeError("libtimebill_kv.so is not built (expected at %s); run "
+                           "paper_2512_21859_gb300.build.build()" % path)
+    lib = ctypes.CDLL(path)
+    P = ctypes.c_void_p
+    I = ctypes.c_int32
+    SZ = ctypes.c_size_t
+    sig = {
+        "tb_status_string": (ctypes.c_char_p, [I]),
+        "tb_abi_version": (I, []),
+        "tb_last_error_detail": (ctypes.c_char_p, []),
+        "tb_launch_counter": (ctypes.c_uint64, []),
+        "tb_retained_count": (I, [ctypes.c_int64, I, ctypes.c_double, _I64P, _I64P]),
+        "tb_evict_layout": (I, [P, _I64P, _I64P]),
+        "tb_evict_workspace_size": (I, [P, ctypes.POINTER(SZ)]),
+        "tb_window_scores": (I, [P, P, P, P, P, SZ, P]),
+        "tb_select_topk": (I, [P, P, P, P, P, SZ, P]),
+        "tb_gather_kv": (I, [P, P, P, P, P, P, P]),
+        "tb_score_evict": (I, [P, P, P, P, P, P, P, P, P, SZ, P]),
+        "tb_decode_workspace_size": (I, [P, ctypes.POINTER(SZ)]),
+        "tb_decode_attn": (I, [P, P, P, P, P, P, P, SZ, P]),
+        "tb_read_status": (I, [P, SZ, P, ctypes.POINTER(I)]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _LIB = lib
+    return lib
+
+
+# ---------------------------------------------------------------------------
+# marshalling helpers
+# ---------------------------------------------------------------------------
+
+def _ptr(x) -> Optional[int]:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        if not x.is_contiguous():
+            raise ValueError("tensor must be contiguous")
+        return x.data_ptr()
+    raise TypeError("expected a tensor, an integer address or None, got %r" % type(x))
+
+
+def _nbytes(x) -> int:
+    return x.numel() * x.element_size()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        if torch.cuda.is_available():
+            return torch.cuda.current_stream().cuda_stream
+        return None
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(status: int, where: str):
+    if status != TB_OK:
+        raise TbError(status, where)
+
+
+class EvictDesc:
+    """tb_evict_desc plus the host arrays it points to (kept alive here)."""
+
+    def __init__(self, *, hq: int, hkv: int, head_dim: int, window: int, pool_k: int,
+                 dtype: int, n: Sequence[int], alpha: Sequence[float],
+                 kv_offset: Optional[Sequence[int]] = None, kv_rows: Optional[int] = None,
+                 out_offset: Optional[Sequence[int]] = None,
+                 out_cap: Optional[Sequence[int]] = None, out_rows: Optional[int] = None,
+                 reserved: int = 0):
+        self.n = np.ascontiguousarray(n, dtype=np.int64)
+        B = self.n.shape[0]
+        self.alpha = np.ascontiguousarray(np.resize(np.asarray(alpha, np.float64), B))
+        if kv_offset is None:
+            kv_offset = np.concatenate([[0], np.cumsum(self.n)[:-1]]) if B else []
+        self.kv_offset = np.ascontiguousarray(kv_offset, dtype=np.int64)
+        if kv_rows is None:
+            kv_rows = int(self.n.sum())
+        if out_cap is None:
+            out_cap = [tb_retained_count(int(nb), window, float(a))[1] if nb >= window >= 1 and 0 <= a <= 1 else 0
+                       for nb, a in zip(self.n, self.alpha)]
+        self.out_cap = np.ascontiguousarray(out_cap, dtype=np.int64)
+        if out_offset is None:
+            out_offset = np.concatenate([[0], np.cumsum(self.out_cap)[:-1]]) if B else []
+        self.out_offset = np.ascontiguousarray(out_offset, dtype=np.int64)
+        if out_rows is None:
+            out_rows = int((self.out_offset + self.out_cap).max()) if B else 0
+        self.hq, self.hkv, self.head_dim, self.window = hq, hkv, head_dim, window
+        self.pool_k, self.dtype = pool_k, dtype
+        self.kv_rows, self.out_rows = int(kv_rows), int(out_rows)
+        self.c = _EvictDescC(
+            B, hq, hkv, head_dim, window, pool_k, dtype, reserved,
+            self.n.ctypes.data_as(_I64P), self.alpha.ctypes.data_as(_F64P),
+            self.kv_offset.ctypes.data_as(_I64P), self.kv_rows,
+            self.out_offset.ctypes.data_as(_I64P), self.out_cap.ctypes.data_as(_I64P),
+            self.out_rows)
+
+    @property
+    def batch(self) -> int:
+        return int(self.n.shape[0])
+
+    def ref(self):
+        return ctypes.byref(self.c)
+
+
+class DecodeDesc:
+    """tb_decode_desc plus its host arrays."""
+
+    def __init__(self, *, hq: int, hkv: int, head_dim: int, dtype: int, cache_offset,
+                 cache_cap, cache_rows: int, max_len: int, out_dtype: int = TB_F32):
+        self.cache_offset = np.ascontiguousarray(cache_offset, dtype=np.int64)
+        self.cache_cap = np.ascontiguousarray(cache_cap, dtype=np.int64)
+        self.c = _DecodeDescC(
+            int(self.cache_offset.shape[0]), hq, hkv, head_dim, dtype, out_dtype,
+            self.cache_offset.ctypes.data_as(_I64P), self.cache_cap.ctypes.data_as(_I64P),
+            int(cache_rows), int(max_len))
+        self.hq, self.hkv, self.head_dim, self.dtype, self.out_dtype = hq, hkv, head_dim, dtype, out_dtype
+        self.cache_rows, self.max_len = int(cache_rows), int(max_len)
+
+    @property
+    def batch(self) -> int:
+        return int(self.cache_offset.shape[0])
+
+    def ref(self):
+        return ctypes.byref(self.c)
+
+
+# ---------------------------------------------------------------------------
+# entry points (same names as the C ABI)
+# ---------------------------------------------------------------------------
+
+def tb_status_string(status: int) -> str:
+    return load().tb_status_string(status).decode()
+
+
+def tb_abi_version() -> int:
+    return load().tb_abi_version()
+
+
+def tb_last_error_detail() -> str:
+    return load().tb_last_error_detail().decode()
+
+
+def tb_launch_counter() -> int:
+    return int(load().tb_launch_counter())
+
+
+def tb_retained_count(n: int, window: int, alpha: float):
+    k = ctypes.c_int64()
+    r = ctypes.c_int64()
+    _check(load().tb_retained_count(int(n), int(window), float(alpha), ctypes.byref(k), ctypes.byref(r)),
+           "tb_retained_count")
+    return k.value, r.value
+
+
+def tb_evict_layout(desc: EvictDesc):
+    s = ctypes.c_int64()
+    i = ctypes.c_int64()
+    _check(load().tb_evict_layout(desc.ref(), ctypes.byref(s), ctypes.byref(i)), "tb_evict_layout")
+    return s.value, i.value
+
+
+def tb_evict_workspace_size(desc: EvictDesc) -> int:
+    b = ctypes.c_size_t()
+    _check(load().tb_evict_workspace_size(desc.ref(), ctypes.byref(b)), "tb_evict_workspace_size")
+    return b.value
+
+
+def _ws(workspace, workspace_bytes):
+    if workspace_bytes is None:
+        workspace_bytes = _nbytes(workspace) if hasattr(workspace, "numel") else 0
+    return _ptr(workspace), workspace_bytes
+
+
+def tb_window_scores(desc: EvictDesc, q_win, K, scores, workspace, workspace_bytes=None, stream=None):
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_window_scores(desc.ref(), _ptr(q_win), _ptr(K), _ptr(scores), w, wb,
+                                   _stream(stream)), "tb_window_scores")
+
+
+def tb_select_topk(desc: EvictDesc, scores, idx, pooled, workspace, workspace_bytes=None, stream=None):
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_select_topk(desc.ref(), _ptr(scores), _ptr(idx), _ptr(pooled), w, wb,
+                                 _stream(stream)), "tb_select_topk")
+
+
+def tb_gather_kv(desc: EvictDesc, idx, K, V, Kc, Vc, stream=None):
+    _check(load().tb_gather_kv(desc.ref(), _ptr(idx), _ptr(K), _ptr(V), _ptr(Kc), _ptr(Vc),
+                               _stream(stream)), "tb_gather_kv")
+
+
+def tb_score_evict(desc: EvictDesc, q_win, K, V, idx, Kc, Vc, pooled, workspace,
+                   workspace_bytes=None, stream=None):
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_score_evict(desc.ref(), _ptr(q_win), _ptr(K), _ptr(V), _ptr(idx), _ptr(Kc),
+                                 _ptr(Vc), _ptr(pooled), w, wb, _stream(stream)), "tb_score_evict")
+
+
+def tb_decode_workspace_size(desc: DecodeDesc) -> int:
+    b = ctypes.c_size_t()
+    _check(load().tb_decode_workspace_size(desc.ref(), ctypes.byref(b)), "tb_decode_workspace_size")
+    return b.value
+
+
+def tb_decode_attn(desc: DecodeDesc, q, Kc, Vc, lens, out, workspace, workspace_bytes=None, stream=None):
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_decode_attn(desc.ref(), _ptr(q), _ptr(Kc), _ptr(Vc), _ptr(lens), _ptr(out), w, wb,
+                                 _stream(stream)), "tb_decode_attn")
+
+
+def tb_read_status(workspace, workspace_bytes=None, stream=None):
+    """Returns (status, raw status word) after waiting for the stream."""
+    w, wb = _ws(workspace, workspace_bytes)
+    raw = ctypes.c_int32()
+    st = load().tb_read_status(w, wb, _stream(stream), ctypes.byref(raw))
+    if st not in (TB_OK, TB_ERR_TIMEOUT, TB_ERR_INVALID_ARG):
+        raise TbError(st, "tb_read_status")
+    return st, raw.value

@@ -1,0 +1,391 @@
+// C-ABI entry points: argument validation, workspace carving, launch order.
+//
+// Every check runs on the host before the first CUDA call, so an invalid
+// call returns without touching the GPU or any output buffer.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+#include <atomic>
+
+#include "tb_internal.cuh"
+
+namespace tb {
+namespace {
+
+thread_local char g_last_error[256] = "";
+std::atomic<uint64_t> g_launches{0};
+
+tb_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return TB_OK;
+  strncpy(g_last_error, cudaGetErrorString(e), sizeof(g_last_error) - 1);
+  g_last_error[sizeof(g_last_error) - 1] = '\0';
+  return TB_ERR_CUDA;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// k = ceil((1 - alpha) n - 1e-9 n), clamped to [0, n - window] (Eq. 8 reading).
+bool retained(int64_t n, int32_t window, double alpha, int64_t* k, int64_t* r) {
+  if (window < 1 || n < window) return false;
+  if (!(alpha >= 0.0 && alpha <= 1.0)) return false;
+  const double x = (1.0 - alpha) * (double)n - 1e-9 * (double)n;
+  int64_t kk = (int64_t)ceil(x);
+  const int64_t p = n - window;
+  if (kk < 0) kk = 0;
+  if (kk > p) kk = p;
+  *k = kk;
+  *r = kk + window;
+  return true;
+}
+
+bool ranges_overlap(const int64_t* off, const int64_t* len, int batch) {
+  for (int a = 0; a < batch; ++a)
+    for (int b = a + 1; b < batch; ++b)
+      if (len[a] > 0 && len[b] > 0 && off[a] < off[b] + len[b] && off[b] < off[a] + len[a])
+        return true;
+  return false;
+}
+
+tb_status build_evict(const tb_evict_desc* d, EvictParams* p) {
+  if (!d) return TB_ERR_INVALID_ARG;
+  if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->window < 1 || d->reserved != 0)
+    return TB_ERR_INVALID_ARG;
+  if (d->batch > TB_MAX_BATCH) return TB_ERR_UNSUPPORTED;
+  if (d->hq % d->hkv != 0) return TB_ERR_INVALID_ARG;
+  if (d->pool_k < 1 || d->pool_k % 2 == 0 || d->pool_k > 63) return TB_ERR_INVALID_ARG;
+  if (d->dtype != TB_F32 && d->dtype != TB_BF16) return TB_ERR_UNSUPPORTED;
+  if (d->head_dim != 64 && d->head_dim != 128) return TB_ERR_UNSUPPORTED;
+  if (!d->n || !d->alpha || !d->kv_offset || !d->out_offset || !d->out_cap)
+    return TB_ERR_INVALID_ARG;
+  if (d->kv_rows < 0 || d->out_rows < 0) return TB_ERR_INVALID_ARG;
+  const int group = d->hq / d->hkv;
+  const int64_t m_rows = (int64_t)group * d->window;
+  if (m_rows > kMaxWindowRows) return TB_ERR_UNSUPPORTED;
+
+  memset(p, 0, sizeof(*p));
+  p->batch = d->batch;
+  p->hq = d->hq;
+  p->hkv = d->hkv;
+  p->group = group;
+  p->d = d->head_dim;
+  p->window = d->window;
+  p->pool_k = d->pool_k;
+  p->dtype = d->dtype;
+  p->m_rows = (int32_t)m_rows;
+  p->chunk = kSimtChunk;
+  p->kv_rows = d->kv_rows;
+  p->out_rows = d->out_rows;
+  p->scale_log2 = (float)(1.4426950408889634 / sqrt((double)d->head_dim));
+
+  int64_t score_rows = 0, idx_rows = 0, items = 0;
+  int64_t rlen[TB_MAX_BATCH];
+  for (int b = 0; b < d->batch; ++b) {
+    const int64_t n = d->n[b];
+    if (n < d->window || n > (int64_t(1) << 30)) return TB_ERR_INVALID_ARG;
+    int64_t k, r;
+    if (!retained(n, d->window, d->alpha[b], &k, &r)) return TB_ERR_INVALID_ARG;
+    if (d->kv_offset[b] < 0 || d->kv_offset[b] + n > d->kv_rows) return TB_ERR_INVALID_ARG;
+    if (d->out_offset[b] < 0 || d->out_cap[b] < r ||
+        d->out_offset[b] + d->out_cap[b] > d->out_rows)
+      return TB_ERR_INVALID_ARG;
+    EvictReq& q = p->req[b];
+    q.kv_off = d->kv_offset[b];
+    q.out_off = d->out_offset[b];
+    q.score_off = score_rows;
+    q.idx_off = idx_rows;
+    q.n = (int32_t)n;
+    q.p = (int32_t)(n - d->window);
+    q.k = (int32_t)k;
+    q.item0 = (int32_t)items;
+    score_rows += n - d->window;
+    idx_rows += r;
+    items += (int64_t)d->hkv * ((n + p->chunk - 1) / p->chunk);
+    if (items > (int64_t)0x7fffffff) return TB_ERR_UNSUPPORTED;
+    p->max_p = std::max<int32_t>(p->max_p, q.p);
+    p->max_r = std::max<int32_t>(p->max_r, (int32_t)r);
+    rlen[b] = d->out_cap[b];
+  }
+  if (ranges_overlap(d->out_offset, rlen, d->batch)) return TB_ERR_INVALID_ARG;
+  p->items = (int32_t)items;
+  p->score_rows = score_rows;
+  p->idx_rows = idx_rows;
+  return TB_OK;
+}
+
+EvictWorkspace carve_evict(const EvictParams& p) {
+  EvictWorkspace w;
+  size_t off = 0;
+  w.status = off;
+  off += kStatusBytes;
+  w.scores = off;
+  off = align_up(off + sizeof(float) * (size_t)p.hkv * p.score_rows, 256);
+  w.partial = off;
+  off = align_up(off + sizeof(float2) * (size_t)p.items * p.m_rows, 256);
+  w.rowc = off;
+  off = align_up(off + sizeof(float) * (size_t)p.batch * p.hkv * p.m_rows, 256);
+  w.pooled = off;
+  off = align_up(off + sizeof(float) * (size_t)p.hkv * p.score_rows, 256);
+  w.total = off;
+  return w;
+}
+
+bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+tb_status check_ws(void* ws, size_t bytes, size_t need) {
+  if (!ws || bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return TB_ERR_WORKSPACE;
+  return TB_OK;
+}
+
+tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
+  if (!d) return TB_ERR_INVALID_ARG;
+  if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->max_len < 1) return TB_ERR_INVALID_ARG;
+  if (d->batch > TB_MAX_BATCH) return TB_ERR_UNSUPPORTED;
+  if (d->hq % d->hkv != 0) return TB_ERR_INVALID_ARG;
+  if (d->dtype != TB_F32 && d->dtype != TB_BF16) return TB_ERR_UNSUPPORTED;
+  if (d->out_dtype != TB_F32 && d->out_dtype != d->dtype) return TB_ERR_UNSUPPORTED;
+  if (d->head_dim != 64 && d->head_dim != 128) return TB_ERR_UNSUPPORTED;
+  if (!d->cache_offset || !d->cache_cap || d->cache_rows < 0) return TB_ERR_INVALID_ARG;
+  if (d->max_len > (int64_t(1) << 30)) return TB_ERR_UNSUPPORTED;
+  const int group = d->hq / d->hkv;
+  const int hs = 128 / d->head_dim;
+  if ((group + hs - 1) / hs > 32) return TB_ERR_UNSUPPORTED;
+  memset(p, 0, sizeof(*p));
+  p->batch = d->batch;
+  p->hq = d->hq;
+  p->hkv = d->hkv;
+  p->group = group;
+  p->d = d->head_dim;
+  p->dtype = d->dtype;
+  p->out_dtype = d->out_dtype;
+  p->cache_rows = d->cache_rows;
+  p->max_len = d->max_len;
+  p->scale_log2 = (float)(1.4426950408889634 / sqrt((double)d->head_dim));
+  for (int b = 0; b < d->batch; ++b) {
+    if (d->cache_offset[b] < 0 || d->cache_cap[b] < 0 ||
+        d->cache_offset[b] + d->cache_cap[b] > d->cache_rows)
+      return TB_ERR_INVALID_ARG;
+    if (d->cache_cap[b] > (int64_t(1) << 30)) return TB_ERR_UNSUPPORTED;
+    p->cache_off[b] = d->cache_offset[b];
+    p->cache_cap[b] = (int32_t)d->cache_cap[b];
+  }
+  // Split the keys so that about four CTAs per SM of a 152-SM part run.
+  const int64_t target = 4 * 152;
+  const int64_t units = (int64_t)d->batch * d->hkv;
+  int64_t splits = (target + units - 1) / units;
+  const int64_t max_splits = (d->max_len + 31) / 32;
+  splits = std::max<int64_t>(1, std::min(splits, max_splits));
+  int64_t split_len = (d->max_len + splits - 1) / splits;
+  split_len = (split_len + 31) / 32 * 32;
+  splits = (d->max_len + split_len - 1) / split_len;
+  p->splits = (int32_t)splits;
+  p->split_len = (int32_t)split_len;
+  return TB_OK;
+}
+
+struct DecodeWorkspace {
+  size_t status, part_o, part_ml, total;
+};
+
+DecodeWorkspace carve_decode(const DecodeParams& p) {
+  DecodeWorkspace w;
+  size_t off = 0;
+  w.status = off;
+  off += kStatusBytes;
+  w.part_o = off;
+  off = align_up(off + sizeof(float) * (size_t)p.batch * p.hq * p.splits * p.d, 256);
+  w.part_ml = off;
+  off = align_up(off + sizeof(float2) * (size_t)p.batch * p.hq * p.splits, 256);
+  w.total = off;
+  return w;
+}
+
+template <typename T>
+T* at(void* base, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(base) + off);
+}
+
+tb_status run_window_scores(const EvictParams& p, const EvictWorkspace& w, const void* q_win,
+                            const void* K, float* scores, void* ws, cudaStream_t s) {
+  return cuda_status(launch_window_scores(p, q_win, K, scores, at<float2>(ws, w.partial),
+                                          at<float>(ws, w.rowc), at<int32_t>(ws, w.status), s));
+}
+
+tb_status run_select(const EvictParams& p, const EvictWorkspace& w, const float* scores,
+                     int32_t* idx, float* pooled, void* ws, cudaStream_t s) {
+  float* pl = pooled ? pooled : at<float>(ws, w.pooled);
+  cudaError_t e = launch_pool(p, scores, pl, s);
+  if (e == cudaSuccess) e = launch_select(p, pl, idx, s);
+  return cuda_status(e);
+}
+
+}  // namespace
+
+void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
+                                 float* scores, float2* partial, float* rowc, int32_t* status,
+                                 cudaStream_t s) {
+  (void)status;
+  return launch_window_scores_simt(p, q_win, K, scores, partial, rowc, s);
+}
+
+}  // namespace tb
+
+using namespace tb;
+
+extern "C" {
+
+const char* tb_status_string(int32_t status) {
+  switch (status) {
+    case TB_OK: return "ok";
+    case TB_ERR_INVALID_ARG: return "invalid argument";
+    case TB_ERR_UNSUPPORTED: return "unsupported configuration";
+    case TB_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case TB_ERR_CUDA: return "CUDA error";
+    case TB_ERR_TIMEOUT: return "device-side wait timed out";
+    default: return "unknown status";
+  }
+}
+
+int32_t tb_abi_version(void) { return 100; }
+
+const char* tb_last_error_detail(void) { return g_last_error; }
+
+uint64_t tb_launch_counter(void) { return g_launches.load(std::memory_order_relaxed); }
+
+tb_status tb_retained_count(int64_t n, int32_t window, double alpha, int64_t* k_out,
+                            int64_t* r_out) {
+  if (!k_out || !r_out) return TB_ERR_INVALID_ARG;
+  int64_t k, r;
+  if (!retained(n, window, alpha, &k, &r)) return TB_ERR_INVALID_ARG;
+  *k_out = k;
+  *r_out = r;
+  return TB_OK;
+}
+
+tb_status tb_evict_layout(const tb_evict_desc* desc, int64_t* score_rows, int64_t* idx_rows) {
+  EvictParams p;
+  const tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  if (score_rows) *score_rows = p.score_rows;
+  if (idx_rows) *idx_rows = p.idx_rows;
+  return TB_OK;
+}
+
+tb_status tb_evict_workspace_size(const tb_evict_desc* desc, size_t* bytes) {
+  if (!bytes) return TB_ERR_INVALID_ARG;
+  EvictParams p;
+  const tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  *bytes = carve_evict(p).total;
+  return TB_OK;
+}
+
+tb_status tb_window_scores(const tb_evict_desc* desc, const void* q_win, const void* K,
+                           float* scores, void* workspace, size_t workspace_bytes,
+                           tb_stream_t stream) {
+  EvictParams p;
+  tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  if (!q_win || !K || !scores || !aligned16(q_win) || !aligned16(K) || !aligned16(scores))
+    return TB_ERR_INVALID_ARG;
+  const EvictWorkspace w = carve_evict(p);
+  if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  return run_window_scores(p, w, q_win, K, scores, workspace, s);
+}
+
+tb_status tb_select_topk(const tb_evict_desc* desc, const float* scores, int32_t* idx,
+                         float* pooled, void* workspace, size_t workspace_bytes,
+                         tb_stream_t stream) {
+  EvictParams p;
+  tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  if (!scores || !idx || !aligned16(scores) || !aligned16(idx) || (pooled && !aligned16(pooled)))
+    return TB_ERR_INVALID_ARG;
+  const EvictWorkspace w = carve_evict(p);
+  if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  return run_select(p, w, scores, idx, pooled, workspace, s);
+}
+
+tb_status tb_gather_kv(const tb_evict_desc* desc, const int32_t* idx, const void* K,
+                       const void* V, void* Kc, void* Vc, tb_stream_t stream) {
+  EvictParams p;
+  const tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  if (!idx || !K || !V || !Kc || !Vc) return TB_ERR_INVALID_ARG;
+  if (!aligned16(idx) || !aligned16(K) || !aligned16(V) || !aligned16(Kc) || !aligned16(Vc))
+    return TB_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return cuda_status(launch_gather(p, idx, K, V, Kc, Vc, s));
+}
+
+tb_status tb_score_evict(const tb_evict_desc* desc, const void* q_win, const void* K,
+                         const void* V, int32_t* idx, void* Kc, void* Vc, float* pooled,
+                         void* workspace, size_t workspace_bytes, tb_stream_t stream) {
+  EvictParams p;
+  tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  if (!q_win || !K || !V || !idx || !Kc || !Vc) return TB_ERR_INVALID_ARG;
+  if (!aligned16(q_win) || !aligned16(K) || !aligned16(V) || !aligned16(idx) ||
+      !aligned16(Kc) || !aligned16(Vc) || (pooled && !aligned16(pooled)))
+    return TB_ERR_INVALID_ARG;
+  const EvictWorkspace w = carve_evict(p);
+  if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  float* scores = at<float>(workspace, w.scores);
+  if ((st = run_window_scores(p, w, q_win, K, scores, workspace, s)) != TB_OK) return st;
+  if ((st = run_select(p, w, scores, idx, pooled, workspace, s)) != TB_OK) return st;
+  return cuda_status(launch_gather(p, idx, K, V, Kc, Vc, s));
+}
+
+tb_status tb_decode_workspace_size(const tb_decode_desc* desc, size_t* bytes) {
+  if (!bytes) return TB_ERR_INVALID_ARG;
+  DecodeParams p;
+  const tb_status st = build_decode(desc, &p);
+  if (st != TB_OK) return st;
+  *bytes = carve_decode(p).total;
+  return TB_OK;
+}
+
+tb_status tb_decode_attn(const tb_decode_desc* desc, const void* q, const void* Kc,
+                         const void* Vc, const int32_t* lens, void* out, void* workspace,
+                         size_t workspace_bytes, tb_stream_t stream) {
+  DecodeParams p;
+  tb_status st = build_decode(desc, &p);
+  if (st != TB_OK) return st;
+  if (!q || !Kc || !Vc || !lens || !out) return TB_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(Kc) || !aligned16(Vc) || !aligned16(out))
+    return TB_ERR_INVALID_ARG;
+  const DecodeWorkspace w = carve_decode(p);
+  if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  return cuda_status(launch_decode(p, q, Kc, Vc, lens, out, at<float>(workspace, w.part_o),
+                                   at<float2>(workspace, w.part_ml),
+                                   at<int32_t>(workspace, w.status), s));
+}
+
+tb_status tb_read_status(const void* workspace, size_t workspace_bytes, tb_stream_t stream,
+                         int32_t* raw) {
+  if (!workspace || workspace_bytes < sizeof(int32_t)) return TB_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  tb_status st = cuda_status(cudaStreamSynchronize(s));
+  if (st != TB_OK) return st;
+  int32_t word = 0;
+  st = cuda_status(cudaMemcpy(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost));
+  if (st != TB_OK) return st;
+  if (raw) *raw = word;
+  if (word & kStatusTimeout) return TB_ERR_TIMEOUT;
+  if (word & kStatusRange) return TB_ERR_INVALID_ARG;
+  return TB_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,104 @@
+// Internal declarations shared by the kernels and the C-ABI layer.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "timebill_kv.h"
+
+namespace tb {
+
+// Bits of the device status word kept at the start of every workspace.
+enum : int32_t {
+  kStatusTimeout = 1,  // a bounded wait gave up
+  kStatusRange = 2,    // a device-side range check fired
+};
+
+// Bytes reserved at the start of each workspace for the status word.
+constexpr size_t kStatusBytes = 256;
+
+// Largest G*W (window rows of one KV-head group) the scoring kernels take.
+constexpr int kMaxWindowRows = 1024;
+
+// Keys per work item of the SIMT scoring kernels.
+constexpr int kSimtChunk = 256;
+
+struct EvictReq {
+  int64_t kv_off;     // first row of the request in K, V
+  int64_t out_off;    // first row in Kc, Vc
+  int64_t score_off;  // first column in scores / pooled
+  int64_t idx_off;    // first column in idx
+  int32_t n;          // prompt length N_b
+  int32_t p;          // prefix length P_b = N_b - W
+  int32_t k;          // retained prefix tokens k_b
+  int32_t item0;      // first work item of the request in the scoring grid
+};
+
+struct EvictParams {
+  int32_t batch, hq, hkv, group, d, window, pool_k, dtype;
+  int32_t m_rows;     // G * W window rows per KV head
+  int32_t chunk;      // keys per scoring work item
+  int32_t items;      // total scoring work items
+  int32_t max_p;      // max_b P_b
+  int32_t max_r;      // max_b R_b
+  int32_t pad0;
+  int64_t kv_rows, out_rows, score_rows, idx_rows;
+  float scale_log2;   // log2(e) / sqrt(d)
+  int32_t pad1;
+  EvictReq req[TB_MAX_BATCH];
+};
+
+struct DecodeParams {
+  int32_t batch, hq, hkv, group, d, dtype, out_dtype, splits;
+  int32_t split_len;  // keys per split
+  int32_t pad0;
+  int64_t cache_rows;
+  int64_t max_len;
+  float scale_log2;
+  int32_t pad1;
+  int64_t cache_off[TB_MAX_BATCH];
+  int32_t cache_cap[TB_MAX_BATCH];
+};
+
+// Workspace carving for the eviction calls (byte offsets, 256-aligned).
+struct EvictWorkspace {
+  size_t status, scores, partial, rowc, pooled, total;
+};
+
+// Adds n to the process-wide launch counter (tb_launch_counter).
+void count_launches(int n);
+
+// ---------------------------------------------------------------------------
+// launchers (each returns cudaGetLastError() of its launch)
+// ---------------------------------------------------------------------------
+cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
+                                 float* scores, float2* partial, float* rowc,
+                                 int32_t* status, cudaStream_t s);
+cudaError_t launch_window_scores_simt(const EvictParams& p, const void* q_win, const void* K,
+                                      float* scores, float2* partial, float* rowc,
+                                      cudaStream_t s);
+cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled,
+                        cudaStream_t s);
+cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* idx,
+                          cudaStream_t s);
+cudaError_t launch_gather(const EvictParams& p, const int32_t* idx, const void* K,
+                          const void* V, void* Kc, void* Vc, cudaStream_t s);
+cudaError_t launch_decode(const DecodeParams& p, const void* q, const void* Kc,
+                          const void* Vc, const int32_t* lens, void* out, float* part_o,
+                          float2* part_ml, int32_t* status, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// device helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float bf16_bits_to_float(uint16_t v) {
+  return __uint_as_float(static_cast<uint32_t>(v) << 16);
+}
+
+template <typename T>
+__device__ __forceinline__ float to_f32(T v);
+template <>
+__device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f32<uint16_t>(uint16_t v) { return bf16_bits_to_float(v); }
+
+}  // namespace tb

@@ -115,8 +115,18 @@ WORKLOADS: Dict[str, Workload] = {
 def f32_to_bf16(x: np.ndarray) -> np.ndarray:
     """Round float32 values to bf16 (nearest, ties to even); returns uint16 bits."""
     b = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
-    rounding = np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1))
-    return ((b + rounding) >> np.uint32(16)).astype(np.uint16)
+    out = np.empty(b.shape, dtype=np.uint16)
+    flat_b, flat_o = b.reshape(-1), out.reshape(-1)
+    step = 1 << 22
+    for s in range(0, flat_b.size, step):
+        chunk = flat_b[s:s + step]
+        r = chunk >> np.uint32(16)
+        r &= np.uint32(1)
+        r += np.uint32(0x7FFF)
+        r += chunk
+        r >>= np.uint32(16)
+        flat_o[s:s + step] = r
+    return out
 
 
 def bf16_to_f32(b: np.ndarray) -> np.ndarray:

@@ -1,0 +1,353 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU fp64 oracle.
+
+Acceptance (the tolerances the method's targets state):
+  * retained index sets bit-exact except positions whose oracle pooled
+    score lies within 1e-6 relative of the k-th largest score;
+  * Kc / Vc bit copies of the rows the GPU selected;
+  * decode attention max-abs error <= 1e-5 for fp32 inputs and <= 2e-2 for
+    bf16 inputs (fp32 accumulation);
+  * window scores within 2e-6 relative (fp32 arithmetic over <= 1024 window
+    rows and one fp32 rounding of each row's log-sum-exp).
+The select and gather stages are also checked alone, bit-exact, on inputs
+the oracle produced (same fp32 scores on both sides).
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from oracle import timebill_oracle as orc  # noqa: E402
+from paper_2512_21859_gb300 import binding as tb  # noqa: E402
+from paper_2512_21859_gb300 import inputs  # noqa: E402
+from tests.gpu_common import (DT, check_index_set, from_dev, request_slices, run_evict,  # noqa: E402
+                              to_dev)
+
+TOL_OUT = {"f32": 1e-5, "bf16": 2e-2}
+TOL_SCORE_REL = 2e-6
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2512_21859_gb300 import build
+    build.build()
+    tb.load()
+
+
+def _f32(wl, x):
+    return inputs.as_f32(x, wl.dtype)
+
+
+def _oracle(wl, lay, heads=None):
+    return orc.score_evict(_f32(wl, lay["q_win"]), _f32(wl, lay["K"]), _f32(wl, lay["V"]),
+                           lay["n"], lay["alpha"], lay["kv_offset"], wl.window, wl.pool_k,
+                           heads=heads)
+
+
+def _check_evict(wl, lay, res, ref, heads=None):
+    desc = res["desc"]
+    K = lay["K"]
+    V = lay["V"]
+    Kc = from_dev(res["Kc_t"], wl.dtype)
+    Vc = from_dev(res["Vc_t"], wl.dtype)
+    excused = 0
+    for b, r in enumerate(ref):
+        s0, i0, P, R = request_slices(desc, b)
+        assert R == r["R"]
+        nb = int(lay["n"][b])
+        for g in (range(wl.hkv) if heads is None else heads):
+            gi = res["idx"][g, i0:i0 + R]
+            excused += check_index_set(gi, r["pooled"][g], r["k"], nb, wl.window)
+            gp = res["pooled"][g, s0:s0 + P].astype(np.float64)
+            if P:
+                np.testing.assert_allclose(gp, r["pooled"][g], rtol=TOL_SCORE_REL, atol=0)
+            off = int(lay["kv_offset"][b])
+            oo = int(desc.out_offset[b])
+            assert np.array_equal(Kc[g, oo:oo + R], K[g, off + gi])
+            assert np.array_equal(Vc[g, oo:oo + R], V[g, off + gi])
+    return excused
+
+
+def _decode_and_check(wl, lay, res, steps, heads_check=None, layer=0):
+    """Appends `steps` decode tokens one by one and checks every step."""
+    desc = res["desc"]
+    B = desc.batch
+    R = [request_slices(desc, b)[3] for b in range(B)]
+    caps = [int(c) for c in desc.out_cap]
+    ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=DT[wl.dtype],
+                          cache_offset=desc.out_offset, cache_cap=caps, cache_rows=desc.out_rows,
+                          max_len=max(R) + steps)
+    ws = torch.empty(tb.tb_decode_workspace_size(ddesc), dtype=torch.uint8, device="cuda")
+    Kc_t, Vc_t = res["Kc_t"], res["Vc_t"]
+    out = torch.empty((B, wl.hq, wl.head_dim), dtype=torch.float32, device="cuda")
+    worst = 0.0
+    for s in range(1, steps + 1):
+        st = inputs.make_decode_step(wl, layer, s, B)
+        kn, vn = to_dev(st["k_new"], wl.dtype), to_dev(st["v_new"], wl.dtype)
+        lens = []
+        for b in range(B):
+            row = int(desc.out_offset[b]) + R[b] + s - 1
+            Kc_t[:, row] = kn[:, b]
+            Vc_t[:, row] = vn[:, b]
+            lens.append(R[b] + s)
+        lens_t = torch.tensor(lens, dtype=torch.int32, device="cuda")
+        q_t = to_dev(st["q"], wl.dtype)
+        tb.tb_decode_attn(ddesc, q_t, Kc_t, Vc_t, lens_t, out, ws)
+        assert tb.tb_read_status(ws)[0] == tb.TB_OK
+        got = out.cpu().numpy()
+        Kc = _f32(wl, from_dev(Kc_t, wl.dtype))
+        Vc = _f32(wl, from_dev(Vc_t, wl.dtype))
+        ref = orc.decode_batch(_f32(wl, st["q"]), Kc, Vc, lens, desc.out_offset)
+        if heads_check is not None:
+            G = wl.group
+            hs = [h for g in heads_check for h in range(g * G, (g + 1) * G)]
+            got, ref = got[:, hs], ref[:, hs]
+        err = float(np.max(np.abs(got - ref)))
+        worst = max(worst, err)
+        assert err <= TOL_OUT[wl.dtype], (s, err)
+    return worst
+
+
+# ---------------------------------------------------------------------------
+# configurations of the method's workloads
+# ---------------------------------------------------------------------------
+
+def test_tiny_config_evict_and_16_decode_steps():
+    wl = inputs.WORKLOADS["tiny"]
+    lay = inputs.make_layer(wl, 0)
+    res = run_evict(wl, lay, extra_cap=wl.decode_steps)
+    ref = _oracle(wl, lay)
+    _check_evict(wl, lay, res, ref)
+    # the GPU selection equals the oracle's exactly here (no in-band ties)
+    assert np.array_equal(res["idx"][:, :ref[0]["R"]], ref[0]["idx"])
+    _decode_and_check(wl, lay, res, wl.decode_steps)
+
+
+@pytest.mark.parametrize("alpha", [0.0, 0.25, 0.5, 0.75])
+def test_7b_config(alpha):
+    wl = inputs.WORKLOADS["7b"]
+    lay = inputs.make_layer(wl, 3, alpha=alpha)
+    res = run_evict(wl, lay, extra_cap=4)
+    ref = _oracle(wl, lay)
+    _check_evict(wl, lay, res, ref)
+    _decode_and_check(wl, lay, res, 2, layer=3)
+
+
+def test_ragged_config():
+    wl = inputs.WORKLOADS["ragged"]
+    lay = inputs.make_layer(wl, 5)
+    res = run_evict(wl, lay, extra_cap=2)
+    ref = _oracle(wl, lay)
+    _check_evict(wl, lay, res, ref)
+    _decode_and_check(wl, lay, res, 2, layer=5)
+
+
+def test_32k_config_alpha_sweep_sampled():
+    """Full-size 32K layer; the oracle scores once and selects per alpha."""
+    wl = inputs.WORKLOADS["32k"]
+    lay = inputs.make_layer(wl, 0)
+    dev = {k: to_dev(lay[k], wl.dtype) for k in ("q_win", "K", "V")}
+    q = _f32(wl, lay["q_win"])[0]
+    K = _f32(wl, lay["K"])
+    S = orc.window_scores(q, K)
+    pooled = orc.max_pool(S, wl.pool_k)
+    n = int(lay["n"][0])
+    for alpha in (0.0, 0.05, 0.5, 0.9, 0.95):
+        lay_a = dict(lay, alpha=np.array([alpha]))
+        res = run_evict(wl, lay_a, extra_cap=1, dev=dev)
+        k, R = orc.retained_count(n, wl.window, alpha)
+        for g in range(wl.hkv):
+            check_index_set(res["idx"][g, :R], pooled[g], k, n, wl.window)
+            np.testing.assert_allclose(res["pooled"][g], pooled[g], rtol=TOL_SCORE_REL, atol=0)
+        if alpha == 0.5:
+            _decode_and_check(wl, lay_a, res, 1)
+
+
+def test_128k_config_sampled_heads():
+    """Full-size 128K layer in the launch configuration the benchmark times;
+    the oracle recomputes KV heads 0 and 7 only."""
+    wl = inputs.WORKLOADS["128k"]
+    lay = inputs.make_layer(wl, 0)
+    res = run_evict(wl, lay, extra_cap=1)
+    ref = _oracle(wl, lay, heads=[0, 7])
+    _check_evict(wl, lay, res, ref, heads=[0, 7])
+    _decode_and_check(wl, lay, res, 1, heads_check=[0, 7])
+
+
+# ---------------------------------------------------------------------------
+# shapes spanning several tiles, ragged tails and the degenerate cases
+# ---------------------------------------------------------------------------
+
+def _custom(dtype, hq, hkv, d, W, pool_k, seed, unit_keys=True, heavy=3):
+    return dataclasses.replace(inputs.WORKLOADS["tiny"], name="custom", hq=hq, hkv=hkv,
+                               head_dim=d, dtype=dtype, window=W, pool_k=pool_k, seed=seed,
+                               unit_keys=unit_keys, heavy_count=heavy, heavy_frac=0.0, batch=1)
+
+
+SHAPES = [
+    # dtype, hq, hkv, d, W, pool_k, n list, alpha list
+    ("f32", 4, 2, 64, 16, 7, [777], [0.5]),
+    ("f32", 3, 3, 128, 5, 3, [1000, 257, 5], [0.3, 0.9, 0.0]),
+    ("bf16", 8, 1, 128, 32, 7, [3001], [0.75]),
+    ("bf16", 7, 1, 64, 8, 13, [2049, 33], [0.1, 1.0]),
+    ("bf16", 28, 4, 128, 32, 7, [1500, 600, 4500], [0.5, 0.0, 0.95]),
+    ("bf16", 4, 4, 128, 64, 1, [640, 64, 65], [0.2, 0.5, 0.5]),   # W = N and W = N - 1
+    ("f32", 2, 1, 64, 1, 63, [300], [0.5]),                       # pool wider than useful
+    ("bf16", 32, 8, 128, 64, 7, [9000], [0.9]),
+]
+
+
+@pytest.mark.parametrize("case", range(len(SHAPES)))
+def test_shapes(case):
+    dtype, hq, hkv, d, W, pk, ns, alphas = SHAPES[case]
+    wl = _custom(dtype, hq, hkv, d, W, pk, seed=100 + case, unit_keys=(dtype == "bf16"))
+    lay = inputs.make_layer(wl, 0, n_override=ns)
+    lay["alpha"] = np.asarray(alphas, dtype=np.float64)
+    res = run_evict(wl, lay, extra_cap=3)
+    ref = _oracle(wl, lay)
+    _check_evict(wl, lay, res, ref)
+    _decode_and_check(wl, lay, res, 3)
+
+
+# ---------------------------------------------------------------------------
+# stages alone, bit-exact on oracle-produced inputs
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_select_stage_exact_on_oracle_scores(seed):
+    rng = np.random.default_rng(seed)
+    W, pk = 16, 7
+    ns = [int(x) for x in rng.integers(W, 20000, size=5)] + [W, W + 1]
+    alphas = list(rng.uniform(0, 1, size=len(ns)))
+    alphas[0] = 0.0
+    alphas[1] = 1.0
+    hkv = 3
+    desc = tb.EvictDesc(hq=hkv, hkv=hkv, head_dim=64, window=W, pool_k=pk, dtype=tb.TB_F32,
+                        n=ns, alpha=alphas)
+    score_rows, idx_rows = tb.tb_evict_layout(desc)
+    # scores with many exact ties (quantised) and a heavy tail
+    S = (np.floor(rng.exponential(1.0, size=(hkv, max(score_rows, 1))) * 64) / 64).astype(np.float32)
+    S_t = torch.from_numpy(S).cuda()
+    idx = torch.full((hkv, idx_rows), -1, dtype=torch.int32, device="cuda")
+    pooled = torch.zeros_like(S_t)
+    ws = torch.empty(tb.tb_evict_workspace_size(desc), dtype=torch.uint8, device="cuda")
+    tb.tb_select_topk(desc, S_t, idx, pooled, ws)
+    gi = idx.cpu().numpy()
+    gp = pooled.cpu().numpy()
+    for b, nb in enumerate(ns):
+        s0, i0, P, R = request_slices(desc, b)
+        k = R - W
+        for g in range(hkv):
+            op = orc.max_pool(S[g, s0:s0 + P].astype(np.float64), pk)
+            assert np.array_equal(gp[g, s0:s0 + P], op.astype(np.float32))
+            assert np.array_equal(gi[g, i0:i0 + R], orc.select_indices(op, k, nb))
+
+
+def test_gather_stage_exact():
+    rng = np.random.default_rng(5)
+    hkv, d, W = 2, 128, 4
+    ns = [300, 1000]
+    desc = tb.EvictDesc(hq=hkv, hkv=hkv, head_dim=d, window=W, pool_k=1, dtype=tb.TB_BF16,
+                        n=ns, alpha=[0.5, 0.25])
+    _, idx_rows = tb.tb_evict_layout(desc)
+    K = rng.integers(0, 1 << 16, size=(hkv, sum(ns), d), dtype=np.uint16)
+    V = rng.integers(0, 1 << 16, size=(hkv, sum(ns), d), dtype=np.uint16)
+    idx = np.zeros((hkv, idx_rows), dtype=np.int32)
+    for b, nb in enumerate(ns):
+        _, i0, P, R = request_slices(desc, b)
+        for g in range(hkv):
+            pick = np.sort(rng.choice(P, size=R - W, replace=False))
+            idx[g, i0:i0 + R] = np.concatenate([pick, np.arange(P, nb)])
+    Kc = torch.zeros((hkv, desc.out_rows, d), dtype=torch.int16, device="cuda")
+    Vc = torch.zeros_like(Kc)
+    tb.tb_gather_kv(desc, torch.from_numpy(idx).cuda(), torch.from_numpy(K.view(np.int16)).cuda(),
+                    torch.from_numpy(V.view(np.int16)).cuda(), Kc, Vc)
+    Kc = Kc.cpu().numpy().view(np.uint16)
+    Vc = Vc.cpu().numpy().view(np.uint16)
+    for b, nb in enumerate(ns):
+        _, i0, P, R = request_slices(desc, b)
+        oo, ko = int(desc.out_offset[b]), int(desc.kv_offset[b])
+        for g in range(hkv):
+            sel = idx[g, i0:i0 + R]
+            assert np.array_equal(Kc[g, oo:oo + R], orc.gather_rows(K[g, ko:ko + nb], sel))
+            assert np.array_equal(Vc[g, oo:oo + R], orc.gather_rows(V[g, ko:ko + nb], sel))
+
+
+@pytest.mark.parametrize("dtype,d,G,out_dtype", [("f32", 64, 2, "f32"), ("bf16", 128, 7, "f32"),
+                                                 ("bf16", 128, 4, "bf16"), ("f32", 128, 1, "f32"),
+                                                 ("bf16", 64, 16, "f32")])
+def test_decode_stage(dtype, d, G, out_dtype):
+    rng = np.random.default_rng(d + G)
+    hkv = 2
+    hq = G * hkv
+    lens = [0, 1, 31, 32, 33, 700, 5000, 2]
+    caps = [max(x, 1) + 5 for x in lens]
+    offs = np.concatenate([[0], np.cumsum(caps)[:-1]])
+    rows = int(np.sum(caps))
+    scale = 1 / np.sqrt(d) if dtype == "bf16" else 1.0
+    Kc = (rng.standard_normal((hkv, rows, d)) * scale).astype(np.float32)
+    Vc = (rng.standard_normal((hkv, rows, d)) * scale).astype(np.float32)
+    q = rng.standard_normal((len(lens), hq, d)).astype(np.float32)
+    store = inputs.f32_to_bf16 if dtype == "bf16" else (lambda x: x)
+    Kc_s, Vc_s, q_s = store(Kc), store(Vc), store(q)
+    ddesc = tb.DecodeDesc(hq=hq, hkv=hkv, head_dim=d, dtype=DT[dtype], cache_offset=offs,
+                          cache_cap=caps, cache_rows=rows, max_len=max(lens),
+                          out_dtype=DT[out_dtype])
+    ws = torch.empty(tb.tb_decode_workspace_size(ddesc), dtype=torch.uint8, device="cuda")
+    odt = torch.float32 if out_dtype == "f32" else torch.bfloat16
+    out = torch.empty((len(lens), hq, d), dtype=odt, device="cuda")
+    tb.tb_decode_attn(ddesc, to_dev(q_s, dtype), to_dev(Kc_s, dtype), to_dev(Vc_s, dtype),
+                      torch.tensor(lens, dtype=torch.int32, device="cuda"), out, ws)
+    assert tb.tb_read_status(ws)[0] == tb.TB_OK
+    got = out.float().cpu().numpy()
+    ref = orc.decode_batch(inputs.as_f32(q_s, dtype), inputs.as_f32(Kc_s, dtype),
+                           inputs.as_f32(Vc_s, dtype), lens, offs)
+    tol = TOL_OUT[dtype] if out_dtype == "f32" else 2e-2
+    assert np.max(np.abs(got - ref)) <= tol
+    assert np.all(got[0] == 0)                     # len 0 writes zeros
+    np.testing.assert_allclose(got[1], np.repeat(inputs.as_f32(Vc_s, dtype)[:, offs[1]], G, axis=0),
+                               atol=tol)           # len 1: the value row itself
+
+
+def test_decode_length_above_cap_is_clamped_and_flagged():
+    rng = np.random.default_rng(9)
+    hkv, G, d = 1, 2, 64
+    caps = [40]
+    Kc = rng.standard_normal((hkv, 40, d)).astype(np.float32)
+    Vc = rng.standard_normal((hkv, 40, d)).astype(np.float32)
+    q = rng.standard_normal((1, G, d)).astype(np.float32)
+    ddesc = tb.DecodeDesc(hq=G, hkv=hkv, head_dim=d, dtype=tb.TB_F32, cache_offset=[0],
+                          cache_cap=caps, cache_rows=40, max_len=64)
+    ws = torch.empty(tb.tb_decode_workspace_size(ddesc), dtype=torch.uint8, device="cuda")
+    out = torch.empty((1, G, d), dtype=torch.float32, device="cuda")
+    tb.tb_decode_attn(ddesc, to_dev(q, "f32"), to_dev(Kc, "f32"), to_dev(Vc, "f32"),
+                      torch.tensor([60], dtype=torch.int32, device="cuda"), out, ws)
+    st, raw = tb.tb_read_status(ws)
+    assert st == tb.TB_ERR_INVALID_ARG and raw & 2
+    ref = orc.decode_batch(q, Kc, Vc, [40], [0])
+    assert np.max(np.abs(out.cpu().numpy() - ref)) <= 1e-5
+    # the next call clears the word
+    tb.tb_decode_attn(ddesc, to_dev(q, "f32"), to_dev(Kc, "f32"), to_dev(Vc, "f32"),
+                      torch.tensor([40], dtype=torch.int32, device="cuda"), out, ws)
+    assert tb.tb_read_status(ws) == (tb.TB_OK, 0)
+
+
+def test_window_scores_stage():
+    wl = _custom("bf16", 28, 4, 128, 32, 7, seed=77)
+    lay = inputs.make_layer(wl, 0, n_override=[5000, 1200])
+    lay["alpha"] = np.array([0.5, 0.5])
+    desc = tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, window=wl.window,
+                        pool_k=wl.pool_k, dtype=tb.TB_BF16, n=lay["n"], alpha=lay["alpha"])
+    score_rows, _ = tb.tb_evict_layout(desc)
+    scores = torch.zeros((wl.hkv, score_rows), dtype=torch.float32, device="cuda")
+    ws = torch.empty(tb.tb_evict_workspace_size(desc), dtype=torch.uint8, device="cuda")
+    tb.tb_window_scores(desc, to_dev(lay["q_win"], "bf16"), to_dev(lay["K"], "bf16"), scores, ws)
+    got = scores.cpu().numpy()
+    ref = _oracle(wl, lay)
+    for b in range(2):
+        s0, _, P, _ = request_slices(desc, b)
+        np.testing.assert_allclose(got[:, s0:s0 + P], ref[b]["S"], rtol=TOL_SCORE_REL, atol=0)
