@@ -1,0 +1,529 @@
+#!/usr/bin/env python
+"""Benchmark of TimeBill's eviction + decode-attention hot path on GB300.
+
+One step = one transformer layer of the path: one decode step of attention
+over the layer's compacted cache (tb_decode_attn), then the layer's
+prompt-time eviction (tb_window_scores -> tb_select_topk -> tb_gather_kv,
+the stages tb_score_evict chains). Layers rotate over enough device buffers
+that every step's inputs are larger than L2 (129 MB), so no step reads
+another step's data from cache; the decode reads a cache the same buffer's
+eviction wrote one rotation earlier.
+
+Prints ONE JSON line. value = algorithmic HBM bytes of the step (K read once
+to score, retained K/V rows read and written, compacted K/V read by decode)
+per second, in GB/s, summed over ranks. Under torchrun every rank runs its
+own replica (independent layers: the path has no cross-rank exchange).
+
+``--impl reference`` times the CPU fp64 oracle instead (the method's only
+reference; no GPU work) on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2512_21859_gb300 import inputs  # noqa: E402
+
+METRIC = "evict + decode-attn µs/layer and HBM GB/s (fraction of ~8 TB/s) vs α"
+L2_BYTES = 129e6
+NOMINAL_HBM_GBS = 8000.0
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="128k", choices=sorted(inputs.WORKLOADS))
+    ap.add_argument("--alpha", type=float, default=None,
+                    help="eviction ratio for every request (default: the workload's own)")
+    ap.add_argument("--sweep", default=None,
+                    help="comma-separated alphas: print one line per alpha")
+    ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target seconds of oracle work for the cpu_baseline sample")
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes (the method's minimum traffic per layer)
+# ---------------------------------------------------------------------------
+
+def elem_bytes(wl):
+    return 4 if wl.dtype == "f32" else 2
+
+
+def retained(n, window, alpha):
+    from paper_2512_21859_gb300 import binding as tb
+    return tb.tb_retained_count(int(n), int(window), float(alpha))
+
+
+def alg_bytes(wl, n, alpha, lens):
+    """Per-layer algorithmic bytes of each stage (HBM, minimum)."""
+    e = elem_bytes(wl)
+    row = e * wl.head_dim
+    B = len(n)
+    R = [retained(nb, wl.window, a)[1] for nb, a in zip(n, alpha)]
+    P = [int(nb) - wl.window for nb in n]
+    q_win = B * wl.hq * wl.window * wl.head_dim * e
+    scores = row * wl.hkv * int(np.sum(n)) + q_win
+    select = 4 * wl.hkv * (2 * int(np.sum(P)) + int(np.sum(R)))
+    gather = 4 * row * wl.hkv * int(np.sum(R))
+    decode = 2 * row * wl.hkv * int(np.sum(lens)) + B * wl.hq * wl.head_dim * (e + 4)
+    evict_min = row * wl.hkv * int(np.sum(n) + 4 * np.sum(R)) + q_win
+    return {"window_scores": scores, "select_topk": select, "gather_kv": gather,
+            "decode_attn": decode, "evict": evict_min, "step": evict_min + decode, "R": R}
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def dist_init(world, use_cuda):
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+    dist.init_process_group(backend="nccl" if use_cuda else "gloo")
+    return dist
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+
+REASONS = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+
+class ClockSampler:
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench_%d.csv" % os.getpid())
+        q = "index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active," + ",".join(
+            "clocks_event_reasons." + r for r in REASONS)
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), "--query-gpu=" + q,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, active = [], [], set()
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 5 + len(REASONS):
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for r, v in zip(REASONS, parts[5:]):
+                    if v.lower().startswith("active"):
+                        active.add(r)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(active)}
+
+
+# ---------------------------------------------------------------------------
+# profile-derived DRAM traffic (ncu), used only while the kernel source matches
+# ---------------------------------------------------------------------------
+
+def kernel_source_digest(files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2512_21859_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(stage, workload):
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        table = json.load(f)
+    ent = table.get("%s/%s" % (stage, workload))
+    if not ent:
+        return None
+    try:
+        if kernel_source_digest(ent["sources"]) != ent["source_digest"]:
+            return None
+    except OSError:
+        return None
+    return ent["dram_bytes_per_launch"]
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args, wl, alpha, world, rank, local, dist):
+    import torch
+    from paper_2512_21859_gb300 import binding as tb
+
+    torch.cuda.set_device(local)
+    tb.load()
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    lay = inputs.make_layer(wl, rank, alpha=alpha)
+    n, a = lay["n"], lay["alpha"]
+    B = len(n)
+    ab = alg_bytes(wl, n, a, [r + 1 for r in [retained(nb, wl.window, x)[1] for nb, x in zip(n, a)]])
+    R = ab["R"]
+    lens_h = [r + 1 for r in R]
+    e = elem_bytes(wl)
+    layer_bytes = 2 * wl.hkv * int(np.sum(n)) * wl.head_dim * e
+    L = int(min(64, max(2, math.ceil(3 * L2_BYTES / layer_bytes))))
+
+    def to_dev(x):
+        if wl.dtype == "bf16":
+            return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+    desc = tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, window=wl.window,
+                        pool_k=wl.pool_k, dtype=tb.TB_BF16 if wl.dtype == "bf16" else tb.TB_F32,
+                        n=n, alpha=a, kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)),
+                        out_cap=[r + 1 for r in R])
+    score_rows, idx_rows = tb.tb_evict_layout(desc)
+    ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
+                          cache_offset=desc.out_offset, cache_cap=desc.out_cap,
+                          cache_rows=desc.out_rows, max_len=max(lens_h))
+    ews = tb.tb_evict_workspace_size(desc)
+    dws = tb.tb_decode_workspace_size(ddesc)
+    step_in = inputs.make_decode_step(wl, rank, 1, B)
+
+    base = {k: to_dev(lay[k]) for k in ("q_win", "K", "V")}
+    q_dec = to_dev(step_in["q"])
+    kn, vn = to_dev(step_in["k_new"]), to_dev(step_in["v_new"])
+    layers = []
+    for li in range(L):
+        d = {k: (v if li == 0 else v.clone()) for k, v in base.items()}
+        d["Kc"] = torch.zeros((wl.hkv, desc.out_rows, wl.head_dim), dtype=base["K"].dtype, device=dev)
+        d["Vc"] = torch.zeros_like(d["Kc"])
+        for b in range(B):   # the decode token's own K/V row, after the retained rows
+            row = int(desc.out_offset[b]) + R[b]
+            d["Kc"][:, row] = kn[:, b]
+            d["Vc"][:, row] = vn[:, b]
+        d["scores"] = torch.empty((wl.hkv, max(score_rows, 1)), dtype=torch.float32, device=dev)
+        d["idx"] = torch.empty((wl.hkv, idx_rows), dtype=torch.int32, device=dev)
+        d["ews"] = torch.empty(ews, dtype=torch.uint8, device=dev)
+        d["dws"] = torch.empty(dws, dtype=torch.uint8, device=dev)
+        d["out"] = torch.empty((B, wl.hq, wl.head_dim), dtype=torch.float32, device=dev)
+        layers.append(d)
+    lens = torch.tensor(lens_h, dtype=torch.int32, device=dev)
+
+    stages = ["decode_attn", "window_scores", "select_topk", "gather_kv"]
+
+    def step(i, evs=None):
+        d = layers[i % L]
+        if evs is not None:
+            evs[0].record(stream)
+        tb.tb_decode_attn(ddesc, q_dec, d["Kc"], d["Vc"], lens, d["out"], d["dws"], stream=stream)
+        if evs is not None:
+            evs[1].record(stream)
+        tb.tb_window_scores(desc, d["q_win"], d["K"], d["scores"], d["ews"], stream=stream)
+        if evs is not None:
+            evs[2].record(stream)
+        tb.tb_select_topk(desc, d["scores"], d["idx"], None, d["ews"], stream=stream)
+        if evs is not None:
+            evs[3].record(stream)
+        tb.tb_gather_kv(desc, d["idx"], d["K"], d["V"], d["Kc"], d["Vc"], stream=stream)
+        if evs is not None:
+            evs[4].record(stream)
+
+    # warm-up: also fills every buffer's compacted cache once
+    for i in range(max(args.warmup, L)):
+        step(i)
+    torch.cuda.synchronize(dev)
+    for d in layers:
+        st, raw = tb.tb_read_status(d["ews"], stream=stream)
+        assert st == tb.TB_OK, raw
+
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    launches0 = tb.tb_launch_counter()
+    t0.record(stream)
+    for i in range(K):
+        step(i, evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    if dist:
+        dist.barrier()
+    launches = tb.tb_launch_counter() - launches0
+    clocks = sampler.stop()
+    total_ms = t0.elapsed_time(t1)
+    if dist:
+        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    for d in layers:
+        st, raw = tb.tb_read_status(d["dws"], stream=stream)
+        assert st == tb.TB_OK, raw
+    stage_ms = {s: sum(ev[j].elapsed_time(ev[j + 1]) for ev in evs) / K for j, s in enumerate(stages)}
+    ms_step = total_ms / K
+    value = world * ab["step"] * K / (total_ms * 1e-3) / 1e9
+
+    # roofline of the dominant stage
+    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+        peaks = json.load(f)
+    peak = float(peaks["hbm_gbs"])
+    dom = max(stages, key=lambda s: stage_ms[s])
+    achieved = ab[dom] / (stage_ms[dom] * 1e-3) / 1e9
+    roof = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+            "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
+            "traffic": profiled_traffic(dom, wl.name),
+            "alg_bytes_per_launch": ab[dom], "avg_launch_ms": round(stage_ms[dom], 5)}
+
+    e2e = run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R)
+
+    evict_us = 1e3 * (stage_ms["window_scores"] + stage_ms["select_topk"] + stage_ms["gather_kv"])
+    res = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
+        "steps": K, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": wl.dtype, "data": "synthetic (seeded Gaussian q/K/V with planted heavy hitters)",
+        "config": {
+            "workload": describe(wl, n, a), "alpha": float(a[0]) if len(set(a.tolist())) == 1 else a.tolist(),
+            "layers_rotated": L, "l2": "inputs larger than L2: %d rotating layer buffers of %.0f MB" % (L, layer_bytes / 1e6),
+            "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
+            "parallelism": "replicas" if world > 1 else "single GPU"},
+        "us_per_layer": {"evict": round(evict_us, 2), "decode": round(1e3 * stage_ms["decode_attn"], 2),
+                         "step": round(1e3 * ms_step, 2),
+                         "stages": {s: round(1e3 * v, 2) for s, v in stage_ms.items()}},
+        "gbs": {"evict": round(ab["evict"] / (evict_us * 1e-6) / 1e9, 1),
+                "decode": round(ab["decode_attn"] / (stage_ms["decode_attn"] * 1e-3) / 1e9, 1)},
+        "frac_of_8tbs": round(value / world / NOMINAL_HBM_GBS, 4),
+        "roofline": roof,
+        "e2e": e2e,
+        "gpu_launches": int(launches),
+        "clocks": clocks,
+    }
+    return res
+
+
+def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R):
+    """The same step through the public API from pinned HOST buffers: every
+    step copies its inputs host->device and reads its results back."""
+    steps = args.e2e_steps if args.e2e_steps is not None else min(args.steps, 10)
+    if steps <= 0:
+        return None
+    B = len(lay["n"])
+
+    def host(x):
+        if wl.dtype == "bf16":
+            t = torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16)
+        else:
+            t = torch.from_numpy(np.ascontiguousarray(x))
+        return t.pin_memory()
+
+    h = {k: host(lay[k]) for k in ("q_win", "K", "V")}
+    hq, hk, hv = host(step_in["q"]), host(step_in["k_new"]), host(step_in["v_new"])
+    d = {k: torch.empty_like(v, device=dev) for k, v in h.items()}
+    qd, kd, vd = torch.empty_like(hq, device=dev), torch.empty_like(hk, device=dev), torch.empty_like(hv, device=dev)
+    score_rows, idx_rows = tb.tb_evict_layout(desc)
+    idx = torch.empty((wl.hkv, idx_rows), dtype=torch.int32, device=dev)
+    Kc = torch.zeros((wl.hkv, desc.out_rows, wl.head_dim), dtype=d["K"].dtype, device=dev)
+    Vc = torch.zeros_like(Kc)
+    ew = torch.empty(ews, dtype=torch.uint8, device=dev)
+    dw = torch.empty(dws, dtype=torch.uint8, device=dev)
+    out = torch.empty((B, wl.hq, wl.head_dim), dtype=torch.float32, device=dev)
+    lens = torch.tensor([r + 1 for r in R], dtype=torch.int32, device=dev)
+    idx_h = torch.empty(idx.shape, dtype=torch.int32).pin_memory()
+    out_h = torch.empty(out.shape, dtype=torch.float32).pin_memory()
+    rows = [int(desc.out_offset[b]) + R[b] for b in range(B)]
+
+    def one():
+        with torch.cuda.stream(stream):
+            for k in d:
+                d[k].copy_(h[k], non_blocking=True)
+            qd.copy_(hq, non_blocking=True)
+            kd.copy_(hk, non_blocking=True)
+            vd.copy_(hv, non_blocking=True)
+            tb.tb_score_evict(desc, d["q_win"], d["K"], d["V"], idx, Kc, Vc, None, ew, stream=stream)
+            for b in range(B):
+                Kc[:, rows[b]] = kd[:, b]
+                Vc[:, rows[b]] = vd[:, b]
+            tb.tb_decode_attn(ddesc, qd, Kc, Vc, lens, out, dw, stream=stream)
+            idx_h.copy_(idx, non_blocking=True)
+            out_h.copy_(out, non_blocking=True)
+
+    for _ in range(2):
+        one()
+    torch.cuda.synchronize(dev)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(steps):
+        one()
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = t0.elapsed_time(t1) / steps
+    h2d = sum(v.numel() * v.element_size() for v in h.values()) + sum(
+        v.numel() * v.element_size() for v in (hq, hk, hv))
+    d2h = idx_h.numel() * 4 + out_h.numel() * 4
+    return {"value": round(ab["step"] / (ms * 1e-3) / 1e9, 1), "unit": "GB/s", "ms_per_step": round(ms, 4),
+            "steps": steps, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+
+def describe(wl, n, a):
+    ns = sorted(set(int(x) for x in n))
+    nd = ("N=%d" % ns[0]) if len(ns) == 1 else ("N in [%d, %d] (%d requests)" % (min(ns), max(ns), len(n)))
+    return "%s: %dq/%dkv heads, d=%d, %s, batch %d, %s, W=%d, pool %d" % (
+        wl.name, wl.hq, wl.hkv, wl.head_dim, wl.dtype, len(n), nd, wl.window, wl.pool_k)
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (cpu_baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(wl, lay, heads, n_keys=None):
+    """Times the oracle on KV heads `heads` of request 0 (optionally on the
+    first n_keys prompt tokens only); returns (seconds, algorithmic bytes)."""
+    from oracle import timebill_oracle as orc
+    q = inputs.as_f32(lay["q_win"], wl.dtype)
+    K = inputs.as_f32(lay["K"], wl.dtype)
+    V = inputs.as_f32(lay["V"], wl.dtype)
+    n = int(lay["n"][0]) if n_keys is None else int(n_keys)
+    a = float(lay["alpha"][0])
+    G = wl.group
+    off = int(lay["kv_offset"][0])
+    e = elem_bytes(wl)
+    row = e * wl.head_dim
+    t0 = time.perf_counter()
+    byt = 0
+    for g in heads:
+        res = orc.score_evict(q[:1, g * G:(g + 1) * G], K[g:g + 1, off:off + n], V[g:g + 1, off:off + n],
+                              [n], [a], [0], wl.window, wl.pool_k)[0]
+        R = res["R"]
+        Kc = np.concatenate([res["Kc"][0], K[g, off + n - 1:off + n]])
+        Vc = np.concatenate([res["Vc"][0], V[g, off + n - 1:off + n]])
+        qd = q[0, g * G:(g + 1) * G, 0]
+        orc.decode_attention(qd, Kc[None], Vc[None], R + 1)
+        byt += row * (n + 4 * R) + G * wl.window * wl.head_dim * e + 2 * row * (R + 1)
+    return time.perf_counter() - t0, byt
+
+
+def cpu_baseline(args, wl, alpha):
+    lay = inputs.make_layer(wl, 0, alpha=alpha)
+    heads, secs, byt = [], 0.0, 0
+    for g in range(wl.hkv):
+        s, b = oracle_sample(wl, lay, [g])
+        heads.append(g)
+        secs += s
+        byt += b
+        if secs >= args.cpu_seconds:
+            break
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {"value": round(byt / secs / 1e9, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "seconds": round(secs, 2),
+            "sample": "eviction of %d of %d KV heads of request 0 of one layer plus one decode step "
+                      "over each head's retained cache, numpy fp64" % (len(heads), wl.hkv)}
+
+
+def run_reference(args, wl, alpha):
+    lay = inputs.make_layer(wl, 0, alpha=alpha)
+    n_full = int(lay["n"][0])
+    # size the per-step sample so that warm-up + steps stay within ~150 s
+    s1, _ = oracle_sample(wl, lay, [0], n_keys=min(n_full, 4096))
+    per_key = s1 / min(n_full, 4096)
+    budget = 150.0 / max(1, args.steps + args.warmup)
+    n_keys = int(min(n_full, max(4 * wl.window, budget / max(per_key, 1e-12))))
+    for i in range(args.warmup):
+        oracle_sample(wl, lay, [i % wl.hkv], n_keys=n_keys)
+    secs, byt = 0.0, 0
+    for i in range(args.steps):
+        s, b = oracle_sample(wl, lay, [i % wl.hkv], n_keys=n_keys)
+        secs += s
+        byt += b
+    value = byt / secs / 1e9
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    sample = ("per step: eviction of one KV head of request 0 over the first %d of %d prompt tokens "
+              "plus one decode step, numpy fp64" % (n_keys, n_full))
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": 0,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * secs / args.steps, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded Gaussian q/K/V with planted heavy hitters)",
+        "config": {"workload": describe(wl, lay["n"], lay["alpha"]), "alpha": float(lay["alpha"][0])},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    world, rank, local = dist_env()
+    wl = inputs.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        print(json.dumps(run_reference(args, wl, args.alpha)), flush=True)
+        return 0
+
+    import torch
+    if not torch.cuda.is_available():
+        print(json.dumps({"error": "no CUDA device: the benchmark times the GPU path only"}))
+        return 1
+    dist = dist_init(world, True)
+    alphas = [float(x) for x in args.sweep.split(",")] if args.sweep else [args.alpha]
+    base_cpu = None
+    for alpha in alphas:
+        res = run_ours(args, wl, alpha, world, rank, local, dist)
+        if rank == 0:
+            if world == 1 and not args.no_cpu_baseline:
+                if base_cpu is None or args.sweep:
+                    base_cpu = cpu_baseline(args, wl, alpha)
+                res["cpu_baseline"] = base_cpu
+            print(json.dumps(res), flush=True)
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
