@@ -210,6 +210,35 @@ tb_status tb_decode_attn(const tb_decode_desc *desc, const void *q,
 tb_status tb_read_status(const void *workspace, size_t workspace_bytes,
                          tb_stream_t stream, int32_t *raw);
 
+/* Size of the device array tb_decode_attn_noalloc uses as its scratch. */
+#define TB_NOALLOC_SCRATCH_BYTES (4u << 20)
+
+/*
+ * tb_decode_attn for callers that cannot allocate device memory (the paper
+ * has no counterpart: this is a deployment convenience). Some callers may not
+ * call an allocator on their per-token path: a hard-real-time loop whose
+ * deadline cannot absorb a cudaMalloc that may synchronise the device, or a
+ * plugin inside a host framework that owns all device memory. This entry
+ * point computes exactly what tb_decode_attn computes, with the same
+ * arguments minus the workspace: its scratch is one library-owned device
+ * array of TB_NOALLOC_SCRATCH_BYTES (4 MiB) that every GPU loading this
+ * library holds until the process exits. It allocates nothing.
+ *  - A descriptor whose tb_decode_workspace_size exceeds the array returns
+ *    TB_ERR_WORKSPACE before any launch; use tb_decode_attn instead.
+ *  - It runs on the calling thread's current device. The first call on each
+ *    device looks up the array's device address there (cudaGetSymbolAddress)
+ *    and keeps it, so make that first call before any stream capture.
+ *  - Every call on a device shares the one array, which keeps the previous
+ *    call's contents: calls that overlap on the GPU (other streams, other
+ *    threads) race and must be serialised by the caller.
+ *  - A length above its cap is clamped as in tb_decode_attn, but the range
+ *    flag cannot be read back (there is no caller workspace to read).
+ */
+tb_status tb_decode_attn_noalloc(const tb_decode_desc *desc, const void *q,
+                                 const void *Kc, const void *Vc,
+                                 const int32_t *lens, void *out,
+                                 tb_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -23,11 +23,13 @@ __all__ = [
     "tb_retained_count", "tb_evict_layout", "tb_evict_workspace_size",
     "tb_window_scores", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
+    "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES",
 ]
 
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
 TB_F32, TB_BF16 = 0, 1
 TB_MAX_BATCH = 64
+TB_NOALLOC_SCRATCH_BYTES = 4 << 20
 
 _I64P = ctypes.POINTER(ctypes.c_int64)
 _F64P = ctypes.POINTER(ctypes.c_double)
@@ -99,6 +101,7 @@ def load():
         "tb_decode_workspace_size": (I, [P, ctypes.POINTER(SZ)]),
         "tb_decode_attn": (I, [P, P, P, P, P, P, P, SZ, P]),
         "tb_read_status": (I, [P, SZ, P, ctypes.POINTER(I)]),
+        "tb_decode_attn_noalloc": (I, [P, P, P, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -291,6 +294,14 @@ def tb_decode_attn(desc: DecodeDesc, q, Kc, Vc, lens, out, workspace, workspace_
     w, wb = _ws(workspace, workspace_bytes)
     _check(load().tb_decode_attn(desc.ref(), _ptr(q), _ptr(Kc), _ptr(Vc), _ptr(lens), _ptr(out), w, wb,
                                  _stream(stream)), "tb_decode_attn")
+
+
+def tb_decode_attn_noalloc(desc: DecodeDesc, q, Kc, Vc, lens, out, stream=None):
+    """tb_decode_attn without a workspace, for callers that cannot allocate
+    device memory: the library's own 4 MiB device array serves as scratch.
+    Calls that overlap on the GPU race on that array."""
+    _check(load().tb_decode_attn_noalloc(desc.ref(), _ptr(q), _ptr(Kc), _ptr(Vc), _ptr(lens), _ptr(out),
+                                         _stream(stream)), "tb_decode_attn_noalloc")
 
 
 def tb_read_status(workspace, workspace_bytes=None, stream=None):

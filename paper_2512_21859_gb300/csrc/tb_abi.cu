@@ -17,12 +17,16 @@ namespace {
 thread_local char g_last_error[256] = "";
 std::atomic<uint64_t> g_launches{0};
 
+}  // namespace
+
 tb_status cuda_status(cudaError_t e) {
   if (e == cudaSuccess) return TB_OK;
   strncpy(g_last_error, cudaGetErrorString(e), sizeof(g_last_error) - 1);
   g_last_error[sizeof(g_last_error) - 1] = '\0';
   return TB_ERR_CUDA;
 }
+
+namespace {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -139,6 +143,8 @@ tb_status check_ws(void* ws, size_t bytes, size_t need) {
   return TB_OK;
 }
 
+}  // namespace
+
 tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
   if (!d) return TB_ERR_INVALID_ARG;
   if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->max_len < 1) return TB_ERR_INVALID_ARG;
@@ -185,10 +191,6 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
   return TB_OK;
 }
 
-struct DecodeWorkspace {
-  size_t status, part_o, part_ml, total;
-};
-
 DecodeWorkspace carve_decode(const DecodeParams& p) {
   DecodeWorkspace w;
   size_t off = 0;
@@ -201,6 +203,8 @@ DecodeWorkspace carve_decode(const DecodeParams& p) {
   w.total = off;
   return w;
 }
+
+namespace {
 
 template <typename T>
 T* at(void* base, size_t off) {

@@ -60,6 +60,18 @@ struct DecodeParams {
   int32_t cache_cap[TB_MAX_BATCH];
 };
 
+// Workspace carving for the decode call (byte offsets, 256-aligned).
+struct DecodeWorkspace {
+  size_t status, part_o, part_ml, total;
+};
+
+// Validates a decode descriptor and fills the kernel parameters.
+tb_status build_decode(const tb_decode_desc* d, DecodeParams* p);
+// Byte layout of the decode workspace for validated parameters.
+DecodeWorkspace carve_decode(const DecodeParams& p);
+// Maps a CUDA error to a status, keeping its text for tb_last_error_detail.
+tb_status cuda_status(cudaError_t e);
+
 // Workspace carving for the eviction calls (byte offsets, 256-aligned).
 struct EvictWorkspace {
   size_t status, scores, partial, rowc, pooled, total;
