@@ -205,6 +205,13 @@ cudaError_t launch_typed(const EvictParams& p, const void* q_win, const void* K,
 
 }  // namespace
 
+cudaError_t launch_window_combine(const EvictParams& p, const float2* partial, float* rowc,
+                                  cudaStream_t s) {
+  ws_combine<<<p.batch * p.hkv, 256, 0, s>>>(p, partial, rowc);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_window_scores_simt(const EvictParams& p, const void* q_win, const void* K,
                                       float* scores, float2* partial, float* rowc,
                                       cudaStream_t s) {

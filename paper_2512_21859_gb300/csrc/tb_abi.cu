@@ -232,7 +232,8 @@ void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order
 cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
                                  float* scores, float2* partial, float* rowc, int32_t* status,
                                  cudaStream_t s) {
-  (void)status;
+  if (window_scores_tc_supported(p))
+    return launch_window_scores_tc(p, q_win, K, scores, partial, rowc, status, s);
   return launch_window_scores_simt(p, q_win, K, scores, partial, rowc, s);
 }
 

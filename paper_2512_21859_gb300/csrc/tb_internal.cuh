@@ -89,6 +89,14 @@ cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const 
 cudaError_t launch_window_scores_simt(const EvictParams& p, const void* q_win, const void* K,
                                       float* scores, float2* partial, float* rowc,
                                       cudaStream_t s);
+// Merges per-chunk (max, sum) partials into one log2-sum-exp per window row.
+cudaError_t launch_window_combine(const EvictParams& p, const float2* partial, float* rowc,
+                                  cudaStream_t s);
+// Tensor-core scoring path (bf16, d in {64, 128}, G*W <= 256).
+bool window_scores_tc_supported(const EvictParams& p);
+cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, const void* K,
+                                    float* scores, float2* partial, float* rowc, int32_t* status,
+                                    cudaStream_t s);
 cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled,
                         cudaStream_t s);
 cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* idx,
