@@ -252,50 +252,77 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
 
     stages = ["decode_attn", "window_scores", "select_topk", "gather_kv"]
 
-    def step(i, evs=None):
-        d = layers[i % L]
-        if evs is not None:
-            evs[0].record(stream)
-        tb.tb_decode_attn(ddesc, q_dec, d["Kc"], d["Vc"], lens, d["out"], d["dws"], stream=stream)
-        if evs is not None:
-            evs[1].record(stream)
-        tb.tb_window_scores(desc, d["q_win"], d["K"], d["scores"], d["ews"], stream=stream)
-        if evs is not None:
-            evs[2].record(stream)
-        tb.tb_select_topk(desc, d["scores"], d["idx"], None, d["ews"], stream=stream)
-        if evs is not None:
-            evs[3].record(stream)
-        tb.tb_gather_kv(desc, d["idx"], d["K"], d["V"], d["Kc"], d["Vc"], stream=stream)
-        if evs is not None:
-            evs[4].record(stream)
+    def stage_call(name, d, st):
+        if name == "decode_attn":
+            tb.tb_decode_attn(ddesc, q_dec, d["Kc"], d["Vc"], lens, d["out"], d["dws"], stream=st)
+        elif name == "window_scores":
+            tb.tb_window_scores(desc, d["q_win"], d["K"], d["scores"], d["ews"], stream=st)
+        elif name == "select_topk":
+            tb.tb_select_topk(desc, d["scores"], d["idx"], None, d["ews"], stream=st)
+        else:
+            tb.tb_gather_kv(desc, d["idx"], d["K"], d["V"], d["Kc"], d["Vc"], stream=st)
 
-    # warm-up: also fills every buffer's compacted cache once
-    for i in range(max(args.warmup, L)):
-        step(i)
+    # eager once per buffer (fills every compacted cache), then capture each
+    # layer's step, and each stage alone, into CUDA graphs
+    for d in layers:
+        for name in stages:
+            stage_call(name, d, stream)
     torch.cuda.synchronize(dev)
     for d in layers:
         st, raw = tb.tb_read_status(d["ews"], stream=stream)
         assert st == tb.TB_OK, raw
+    cap = torch.cuda.Stream(dev)
+    step_graphs, stage_graphs = [], []
+    kernels_per_step = None
+    for d in layers:
+        g = torch.cuda.CUDAGraph()
+        c0 = tb.tb_launch_counter()
+        with torch.cuda.graph(g, stream=cap):
+            for name in stages:
+                stage_call(name, d, cap)
+        kernels_per_step = tb.tb_launch_counter() - c0
+        step_graphs.append(g)
+        per = []
+        for name in stages:
+            gs = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gs, stream=cap):
+                stage_call(name, d, cap)
+            per.append(gs)
+        stage_graphs.append(per)
+    torch.cuda.synchronize(dev)
+
+    with torch.cuda.stream(stream):
+        for i in range(max(args.warmup, L)):
+            step_graphs[i % L].replay()
+    torch.cuda.synchronize(dev)
 
     K = args.steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local)
     if dist:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    launches0 = tb.tb_launch_counter()
-    t0.record(stream)
-    for i in range(K):
-        step(i, evs[i])
-    t1.record(stream)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for i in range(K):
+            step_graphs[i % L].replay()
+        t1.record(stream)
     torch.cuda.synchronize(dev)
     if dist:
         dist.barrier()
-    launches = tb.tb_launch_counter() - launches0
-    clocks = sampler.stop()
     total_ms = t0.elapsed_time(t1)
+    # the same steps once more, stage by stage, with events between stages
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    with torch.cuda.stream(stream):
+        for i in range(K):
+            evs[i][0].record(stream)
+            for j in range(4):
+                stage_graphs[i % L][j].replay()
+                evs[i][j + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = sampler.stop()
+    launches = kernels_per_step * K
     if dist:
         t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -330,6 +357,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             "workload": describe(wl, n, a), "alpha": float(a[0]) if len(set(a.tolist())) == 1 else a.tolist(),
             "layers_rotated": L, "l2": "inputs larger than L2: %d rotating layer buffers of %.0f MB" % (L, layer_bytes / 1e6),
             "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
+            "launch": "each step is one CUDA-graph replay of the four C-ABI calls; stage times from per-stage graph replays with events between them",
             "parallelism": "replicas" if world > 1 else "single GPU"},
         "us_per_layer": {"evict": round(evict_us, 2), "decode": round(1e3 * stage_ms["decode_attn"], 2),
                          "step": round(1e3 * ms_step, 2),
@@ -340,6 +368,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         "roofline": roof,
         "e2e": e2e,
         "gpu_launches": int(launches),
+        "gpu_launches_per_step": int(kernels_per_step),
         "clocks": clocks,
     }
     return res

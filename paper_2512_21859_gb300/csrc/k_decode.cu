@@ -19,13 +19,6 @@ namespace {
 constexpr int kDecThreads = 128;
 constexpr int kTile = 32;
 
-__device__ __forceinline__ uint16_t float_to_bf16_rne(float f) {
-  uint32_t u = __float_as_uint(f);
-  if ((u & 0x7f800000u) == 0x7f800000u) return static_cast<uint16_t>(u >> 16 | ((u & 0xffffu) ? 0x40u : 0u));
-  u += 0x7fffu + ((u >> 16) & 1u);
-  return static_cast<uint16_t>(u >> 16);
-}
-
 __device__ __forceinline__ int clamp_len(const DecodeParams& p, const int32_t* lens, int b,
                                          int32_t* status, bool report) {
   int len = lens[b];
@@ -204,7 +197,9 @@ cudaError_t launch_d(const DecodeParams& p, const void* q, const void* Kc, const
 
 cudaError_t launch_decode(const DecodeParams& p, const void* q, const void* Kc, const void* Vc,
                           const int32_t* lens, void* out, float* part_o, float2* part_ml,
-                          int32_t* status, cudaStream_t s) {
+                          int32_t* counters, int32_t* status, cudaStream_t s) {
+  if (decode_tma_supported(p))
+    return launch_decode_tma(p, q, Kc, Vc, lens, part_o, part_ml, counters, out, status, s);
   if (p.dtype == TB_F32) {
     return p.d == 64 ? launch_d<float, 64>(p, q, Kc, Vc, lens, out, part_o, part_ml, status, s)
                      : launch_d<float, 128>(p, q, Kc, Vc, lens, out, part_o, part_ml, status, s);

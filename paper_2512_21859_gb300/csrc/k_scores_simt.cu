@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(256) ws_stats_simt(const __grid_constant__ Evi
   }
 }
 
-// (2) merge chunk partials: c = m + log2(l), in double precision.
+// (2) merge chunk partials: c = m + log2(l), fp32 with a compensated sum.
 __global__ void __launch_bounds__(256) ws_combine(const __grid_constant__ EvictParams p,
                                                   const float2* __restrict__ partial,
                                                   float* __restrict__ rowc) {
@@ -121,14 +121,19 @@ __global__ void __launch_bounds__(256) ws_combine(const __grid_constant__ EvictP
   const int M = p.m_rows;
   const size_t item0 = (size_t)rq.item0 + (size_t)g * nch;
   for (int r = threadIdx.x; r < M; r += blockDim.x) {
-    double m = -INFINITY;
-    for (int c = 0; c < nch; ++c) m = fmax(m, (double)partial[(item0 + c) * M + r].x);
-    double l = 0.0;
+    float m = -INFINITY;
+    for (int c = 0; c < nch; ++c) m = fmaxf(m, partial[(item0 + c) * M + r].x);
+    float l = 0.f, comp = 0.f;  // compensated (Kahan) sum
     for (int c = 0; c < nch; ++c) {
       const float2 v = partial[(item0 + c) * M + r];
-      if (v.y > 0.f) l += (double)v.y * exp2((double)v.x - m);
+      if (v.y > 0.f) {
+        const float term = v.y * exp2f(v.x - m) - comp;
+        const float t = l + term;
+        comp = (t - l) - term;
+        l = t;
+      }
     }
-    rowc[(size_t)seg * M + r] = (float)(m + log2(l));
+    rowc[(size_t)seg * M + r] = m + log2f(l);
   }
 }
 

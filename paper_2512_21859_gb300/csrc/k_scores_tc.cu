@@ -232,7 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int vis_end = min(rq.n, rq.p + w + 1);  // keys [0, vis_end) visible to the row
     const float c = p.scale_log2;
     float m_run = -INFINITY;
-    double l_run = 0.0;
+    float l_run = 0.f, l_comp = 0.f;  // compensated running sum of 2^(t - m_run)
     bool ok = true;
     for (int it = 0; it < ntiles; ++it) {
       const int a = it & 1;
@@ -262,7 +262,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float m_new = fmaxf(m_run, mx * c);
           if (m_new != -INFINITY) {  // some key of this chunk is visible
             if (m_new > m_run) {
-              l_run *= (double)fast_exp2(m_run - m_new);
+              const float sc = fast_exp2(m_run - m_new);
+              l_run *= sc;
+              l_comp *= sc;
               m_run = m_new;
             }
             float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
@@ -273,7 +275,10 @@ __global__ void __launch_bounds__(kThreads, 1)
               s2 += fast_exp2(fmaf(v[i + 2], c, -m_run));
               s3 += fast_exp2(fmaf(v[i + 3], c, -m_run));
             }
-            l_run += (double)((s0 + s1) + (s2 + s3));
+            const float term = ((s0 + s1) + (s2 + s3)) - l_comp;
+            const float tsum = l_run + term;
+            l_comp = (tsum - l_run) - term;
+            l_run = tsum;
           }
         }
       }
@@ -281,7 +286,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
     }
-    if (ok && wg < RB && row < M) partial[(size_t)item * M + row] = make_float2(m_run, (float)l_run);
+    if (ok && wg < RB && row < M) partial[(size_t)item * M + row] = make_float2(m_run, l_run);
   }
   teardown(bars, tmem, issued, committed, status);
 }
@@ -434,19 +439,27 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 2-D bf16 map over rows of `d` elements: boxes of 128 rows x 64 columns,
-// 128-byte swizzle (the layout the MMA descriptors expect).
 bool make_map(CUtensorMap* map, const void* base, int d, uint64_t rows) {
+  return make_bf16_map(map, base, d, rows, 128);
+}
+
+}  // namespace
+
+// 2-D bf16 map over rows of `d` elements: boxes of box_rows rows x 64
+// columns, 128-byte swizzle (the layout the MMA descriptors expect).
+bool make_bf16_map(CUtensorMap* map, const void* base, int d, uint64_t rows, int box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)d * 2};
-  cuuint32_t box[2] = {64, 128};
+  cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
+
+namespace {
 
 template <int D>
 cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const CUtensorMap& tk,

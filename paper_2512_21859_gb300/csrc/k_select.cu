@@ -11,6 +11,7 @@
 // tau-valued entries to keep; one ordered pass then keeps every entry above
 // tau and the first `need` entries equal to tau, which yields sorted indices
 // without a sort.
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
 #include "tb_internal.cuh"
@@ -149,6 +150,206 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Cluster select: one thread-block cluster of `cs` CTAs per (request, KV head)
+// segment. CTA r of the cluster owns prefix positions [r*L, r*L + L): it loads
+// that slice of the scores with a pool_k/2 halo into shared memory, max-pools
+// it in place, and keeps the pooled bit patterns there. The four radix passes
+// build a 256-bin histogram per CTA; every CTA sums the cluster's histograms
+// through distributed shared memory and derives the same digit. Compaction
+// runs warp by warp over contiguous runs with ballots, after one exchange of
+// per-CTA (greater, equal) counts fixes each CTA's output offset.
+// ---------------------------------------------------------------------------
+constexpr int kCsThreads = 1024;
+constexpr int kCsWarps = kCsThreads / 32;
+
+struct ClusterSelectShared {
+  unsigned hist[2][256];
+  unsigned total[256];
+  int wgt[kCsWarps], weq[kCsWarps];
+  int cta_cnt[2];  // this CTA's (greater, equal) counts, read by the cluster
+  unsigned prefix;
+  int need;
+};
+
+__global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
+    const __grid_constant__ EvictParams p, const float* __restrict__ scores,
+    float* __restrict__ pooled_out, int32_t* __restrict__ idx, int slice) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
+  __shared__ ClusterSelectShared sh;
+  extern __shared__ float keys_f[];  // slice + 2 * halo floats
+  unsigned* keys = reinterpret_cast<unsigned*>(keys_f);
+
+  const int cs = (int)cluster.num_blocks();
+  const int rank = (int)cluster.block_rank();
+  const int seg = blockIdx.x / cs;
+  const int b = seg / p.hkv, g = seg % p.hkv;
+  const EvictReq& rq = p.req[b];
+  const int P = rq.p, k = rq.k, half = p.pool_k / 2;
+  const int lo = min(P, rank * slice);
+  const int cnt = max(0, min(P, lo + slice) - lo);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* S = scores + (size_t)g * p.score_rows + rq.score_off;
+  int32_t* out = idx + (size_t)g * p.idx_rows + rq.idx_off;
+
+  if (rank == 0)
+    for (int t = tid; t < p.window; t += kCsThreads) out[k + t] = P + t;
+
+  // slice + halo, -inf outside the prefix (scores are >= 0, so max is exact)
+  for (int i = tid; i < cnt + 2 * half; i += kCsThreads) {
+    const int j = lo - half + i;
+    keys_f[i] = (j >= 0 && j < P) ? S[j] : -INFINITY;
+  }
+  __syncthreads();
+  constexpr int kMaxPer = kClusterSliceMax / kCsThreads;
+  unsigned reg[kMaxPer];
+#pragma unroll
+  for (int r = 0; r < kMaxPer; ++r) {
+    const int i = tid + r * kCsThreads;
+    if (i < cnt) {
+      float m = keys_f[i];
+      for (int t = 1; t <= 2 * half; ++t) m = fmaxf(m, keys_f[i + t]);
+      reg[r] = __float_as_uint(m);
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < kMaxPer; ++r) {
+    const int i = tid + r * kCsThreads;
+    if (i < cnt) keys[i] = reg[r];
+  }
+  __syncthreads();
+  if (pooled_out) {
+    float* po = pooled_out + (size_t)g * p.score_rows + rq.score_off + lo;
+    for (int i = tid; i < cnt; i += kCsThreads) po[i] = __uint_as_float(keys[i]);
+  }
+
+  // ---- radix select of the k-th largest key (uniform across the cluster)
+  unsigned tau = 0;
+  int need = 0;
+  const bool partial_sel = k > 0 && k < P;
+  if (partial_sel) {
+    unsigned prefix = 0, mask = 0;
+    need = k;
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      unsigned* h = sh.hist[pass & 1];
+      for (int t = tid; t < 256; t += kCsThreads) h[t] = 0;
+      __syncthreads();
+      for (int i = tid; i - lane < cnt; i += kCsThreads) {
+        const bool valid = i < cnt && ((keys[i < cnt ? i : 0] & mask) == prefix);
+        const unsigned dg = valid ? (keys[i] >> shift) & 255u : 256u;
+        const unsigned d0 = __shfl_sync(0xffffffffu, dg, 0);
+        if (__all_sync(0xffffffffu, dg == d0)) {
+          if (lane == 0 && d0 < 256u) atomicAdd(&h[d0], 32u);
+        } else if (valid) {
+          atomicAdd(&h[dg], 1u);
+        }
+      }
+      cluster.sync();
+      for (int t = tid; t < 256; t += kCsThreads) {
+        unsigned sum = 0;
+        for (int r = 0; r < cs; ++r) sum += cluster.map_shared_rank(h, r)[t];
+        sh.total[t] = sum;
+      }
+      __syncthreads();
+      if (warp == 0) {
+        unsigned cntd[8], mine = 0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          cntd[i] = sh.total[255 - (lane * 8 + i)];
+          mine += cntd[i];
+        }
+        unsigned inc = mine;
+        for (int off = 1; off < 32; off <<= 1) {
+          const unsigned o = __shfl_up_sync(0xffffffffu, inc, off);
+          if (lane >= off) inc += o;
+        }
+        const unsigned above = inc - mine;
+        if (above < (unsigned)need && inc >= (unsigned)need) {
+          unsigned run = above;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            if (run + cntd[i] >= (unsigned)need) {
+              sh.prefix = prefix | ((255u - (unsigned)(lane * 8 + i)) << shift);
+              sh.need = need - (int)run;
+              break;
+            }
+            run += cntd[i];
+          }
+        }
+      }
+      __syncthreads();
+      prefix = sh.prefix;
+      need = sh.need;
+      mask |= 255u << shift;
+    }
+    tau = prefix;
+  } else if (k >= P) {
+    tau = 0u;  // keep everything: every key is >= +0.0
+    need = P;
+  }
+
+  // ---- ordered compaction over warp-contiguous runs
+  const int run = ((cnt + kCsWarps - 1) / kCsWarps + 31) & ~31;
+  const int wlo = min(cnt, warp * run), whi = min(cnt, wlo + run);
+  int gt_w = 0, eq_w = 0;
+  if (k > 0) {
+    for (int base = wlo; base < whi; base += 32) {
+      const int i = base + lane;
+      const unsigned u = i < whi ? keys[i] : 0u;
+      gt_w += __popc(__ballot_sync(0xffffffffu, i < whi && u > tau));
+      eq_w += __popc(__ballot_sync(0xffffffffu, i < whi && u == tau));
+    }
+  }
+  if (lane == 0) {
+    sh.wgt[warp] = gt_w;
+    sh.weq[warp] = eq_w;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int gsum = 0, esum = 0;
+    for (int w = 0; w < kCsWarps; ++w) {
+      gsum += sh.wgt[w];
+      esum += sh.weq[w];
+    }
+    sh.cta_cnt[0] = gsum;
+    sh.cta_cnt[1] = esum;
+  }
+  cluster.sync();
+  // offsets of this CTA: ties are kept in index order until `need` are in
+  int eqbase = 0, selbase = 0;
+  for (int r = 0; r < rank; ++r) {
+    const int* c = cluster.map_shared_rank(sh.cta_cnt, r);
+    const int tg = c[0], te = c[1];
+    selbase += tg + max(0, min(need - eqbase, te));
+    eqbase += te;
+  }
+  for (int w = 0; w < warp; ++w) {
+    selbase += sh.wgt[w] + max(0, min(need - eqbase, sh.weq[w]));
+    eqbase += sh.weq[w];
+  }
+  if (k > 0) {
+    const unsigned lt = (1u << lane) - 1u;
+    for (int base = wlo; base < whi; base += 32) {
+      const int i = base + lane;
+      const unsigned u = i < whi ? keys[i] : 0u;
+      const bool gt = i < whi && u > tau;
+      const bool eq = i < whi && u == tau;
+      const unsigned em = __ballot_sync(0xffffffffu, eq);
+      const bool sel = gt || (eq && eqbase + __popc(em & lt) < need);
+      const unsigned sm = __ballot_sync(0xffffffffu, sel);
+      const int pos = selbase + __popc(sm & lt);
+      if (sel && pos < k) out[pos] = lo + i;
+      selbase += __popc(sm);
+      eqbase += __popc(em);
+    }
+  }
+  cluster.sync();  // no CTA leaves while another may still read its shared memory
+}
+
 }  // namespace
 
 cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled, cudaStream_t s) {
@@ -164,6 +365,43 @@ cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* id
                           cudaStream_t s) {
   select_kernel<<<p.batch * p.hkv, kSelThreads, 0, s>>>(p, pooled, idx);
   count_launches(1);
+  return cudaGetLastError();
+}
+
+bool select_cluster_supported(const EvictParams& p) {
+  const int cs = select_cluster_size(p);
+  const int slice = (p.max_p + cs - 1) / cs;
+  return slice <= kClusterSliceMax;
+}
+
+int select_cluster_size(const EvictParams& p) {
+  int cs = (p.max_p + 8191) / 8192;
+  return cs < 1 ? 1 : (cs > 8 ? 8 : cs);
+}
+
+cudaError_t launch_select_cluster(const EvictParams& p, const float* scores, float* pooled_out,
+                                  int32_t* idx, cudaStream_t s) {
+  const int cs = select_cluster_size(p);
+  const int slice = (p.max_p + cs - 1) / cs;
+  const size_t smem = sizeof(float) * ((size_t)slice + 2 * (p.pool_k / 2));
+  cudaError_t e = cudaFuncSetAttribute(select_cluster_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(p.batch * p.hkv * cs), 1, 1);
+  cfg.blockDim = dim3(kCsThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, select_cluster_kernel, p, scores, pooled_out, idx, slice);
+  count_launches(1);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

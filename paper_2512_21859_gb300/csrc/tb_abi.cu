@@ -177,14 +177,15 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
     p->cache_off[b] = d->cache_offset[b];
     p->cache_cap[b] = (int32_t)d->cache_cap[b];
   }
-  // Split the keys so that about four CTAs per SM of a 152-SM part run.
-  const int64_t target = 4 * 152;
+  // Split the keys so that about two CTAs per SM of a 152-SM part run, in
+  // whole 64-key tiles.
+  const int64_t target = 2 * 152;
   const int64_t units = (int64_t)d->batch * d->hkv;
   int64_t splits = (target + units - 1) / units;
-  const int64_t max_splits = (d->max_len + 31) / 32;
+  const int64_t max_splits = (d->max_len + 63) / 64;
   splits = std::max<int64_t>(1, std::min(splits, max_splits));
   int64_t split_len = (d->max_len + splits - 1) / splits;
-  split_len = (split_len + 31) / 32 * 32;
+  split_len = (split_len + 63) / 64 * 64;
   splits = (d->max_len + split_len - 1) / split_len;
   p->splits = (int32_t)splits;
   p->split_len = (int32_t)split_len;
@@ -196,6 +197,8 @@ DecodeWorkspace carve_decode(const DecodeParams& p) {
   size_t off = 0;
   w.status = off;
   off += kStatusBytes;
+  w.counters = off;
+  off = align_up(off + sizeof(int32_t) * (size_t)p.batch * p.hkv, 256);
   w.part_o = off;
   off = align_up(off + sizeof(float) * (size_t)p.batch * p.hq * p.splits * p.d, 256);
   w.part_ml = off;
@@ -219,6 +222,7 @@ tb_status run_window_scores(const EvictParams& p, const EvictWorkspace& w, const
 
 tb_status run_select(const EvictParams& p, const EvictWorkspace& w, const float* scores,
                      int32_t* idx, float* pooled, void* ws, cudaStream_t s) {
+  if (select_cluster_supported(p)) return cuda_status(launch_select_cluster(p, scores, pooled, idx, s));
   float* pl = pooled ? pooled : at<float>(ws, w.pooled);
   cudaError_t e = launch_pool(p, scores, pl, s);
   if (e == cudaSuccess) e = launch_select(p, pl, idx, s);
@@ -372,9 +376,10 @@ tb_status tb_decode_attn(const tb_decode_desc* desc, const void* q, const void* 
   const DecodeWorkspace w = carve_decode(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, w.part_o, s))) != TB_OK) return st;
   return cuda_status(launch_decode(p, q, Kc, Vc, lens, out, at<float>(workspace, w.part_o),
                                    at<float2>(workspace, w.part_ml),
+                                   at<int32_t>(workspace, w.counters),
                                    at<int32_t>(workspace, w.status), s));
 }
 

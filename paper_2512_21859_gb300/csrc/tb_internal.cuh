@@ -1,6 +1,7 @@
 // Internal declarations shared by the kernels and the C-ABI layer.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -62,7 +63,7 @@ struct DecodeParams {
 
 // Workspace carving for the decode call (byte offsets, 256-aligned).
 struct DecodeWorkspace {
-  size_t status, part_o, part_ml, total;
+  size_t status, counters, part_o, part_ml, total;  // [0, part_o) is zeroed per call
 };
 
 // Validates a decode descriptor and fills the kernel parameters.
@@ -76,6 +77,10 @@ tb_status cuda_status(cudaError_t e);
 struct EvictWorkspace {
   size_t status, scores, partial, rowc, pooled, total;
 };
+
+// 2-D bf16 TMA map over rows of d elements, boxes of box_rows x 64 columns
+// with 128-byte swizzle; false if the driver entry point is missing.
+bool make_bf16_map(CUtensorMap* map, const void* base, int d, uint64_t rows, int box_rows);
 
 // Adds n to the process-wide launch counter (tb_launch_counter).
 void count_launches(int n);
@@ -101,17 +106,38 @@ cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled
                         cudaStream_t s);
 cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* idx,
                           cudaStream_t s);
+// Cluster select with the max-pool fused in (pooled_out may be null).
+constexpr int kClusterSliceMax = 16 * 1024;  // keys per CTA: 16 per thread of 1024
+int select_cluster_size(const EvictParams& p);
+bool select_cluster_supported(const EvictParams& p);
+cudaError_t launch_select_cluster(const EvictParams& p, const float* scores, float* pooled_out,
+                                  int32_t* idx, cudaStream_t s);
 cudaError_t launch_gather(const EvictParams& p, const int32_t* idx, const void* K,
                           const void* V, void* Kc, void* Vc, cudaStream_t s);
+// TMA-staged bf16 decode (split partials only; the caller launches the combine).
+bool decode_tma_supported(const DecodeParams& p);
+cudaError_t launch_decode_tma(const DecodeParams& p, const void* q, const void* Kc,
+                              const void* Vc, const int32_t* lens, float* part_o,
+                              float2* part_ml, int32_t* counters, void* out, int32_t* status,
+                              cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, const void* q, const void* Kc,
                           const void* Vc, const int32_t* lens, void* out, float* part_o,
-                          float2* part_ml, int32_t* status, cudaStream_t s);
+                          float2* part_ml, int32_t* counters, int32_t* status, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // device helpers
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float bf16_bits_to_float(uint16_t v) {
   return __uint_as_float(static_cast<uint32_t>(v) << 16);
+}
+
+// fp32 -> bf16 bits, round to nearest even (NaN stays NaN).
+__device__ __forceinline__ uint16_t float_to_bf16_rne(float f) {
+  uint32_t u = __float_as_uint(f);
+  if ((u & 0x7f800000u) == 0x7f800000u)
+    return static_cast<uint16_t>((u >> 16) | ((u & 0xffffu) ? 0x40u : 0u));
+  u += 0x7fffu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>(u >> 16);
 }
 
 template <typename T>

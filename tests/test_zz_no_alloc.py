@@ -51,8 +51,8 @@ def _dev(x, dtype):
 
 
 def test_oversized_descriptor_is_rejected_before_launch(lib):
-    # 64 requests x 64 heads x many splits of partials: far beyond 4 MiB
-    desc = tb.DecodeDesc(hq=64, hkv=8, head_dim=128, dtype=tb.TB_BF16, cache_offset=np.arange(64) * 100000,
+    # 64 requests x 128 query heads x d 128 of fp32 split partials: beyond 4 MiB
+    desc = tb.DecodeDesc(hq=128, hkv=8, head_dim=128, dtype=tb.TB_BF16, cache_offset=np.arange(64) * 100000,
                          cache_cap=[100000] * 64, cache_rows=6400000, max_len=100000)
     assert tb.tb_decode_workspace_size(desc) > tb.TB_NOALLOC_SCRATCH_BYTES
     fake = 1 << 20
