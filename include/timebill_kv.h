@@ -210,6 +210,14 @@ tb_status tb_decode_attn(const tb_decode_desc *desc, const void *q,
 tb_status tb_read_status(const void *workspace, size_t workspace_bytes,
                          tb_stream_t stream, int32_t *raw);
 
+/*
+ * Diagnostic: y[i] = 2^x[i] computed by the FMA-pipe exponential the scoring
+ * kernels use for part of their softmax terms (Cody-Waite range reduction and
+ * a degree-5 polynomial; relative error below 2.2e-7 for x in [-125, 0.5];
+ * inputs below -125 are clamped there). x, y: device float arrays of n.
+ */
+tb_status tb_diag_exp2(const float *x, float *y, int64_t n, tb_stream_t stream);
+
 /* Size of the device array tb_decode_attn_noalloc uses as its scratch. */
 #define TB_NOALLOC_SCRATCH_BYTES (4u << 20)
 

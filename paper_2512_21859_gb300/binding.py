@@ -23,7 +23,7 @@ __all__ = [
     "tb_retained_count", "tb_evict_layout", "tb_evict_workspace_size",
     "tb_window_scores", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
-    "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES",
+    "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_exp2",
 ]
 
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
@@ -102,6 +102,7 @@ def load():
         "tb_decode_attn": (I, [P, P, P, P, P, P, P, SZ, P]),
         "tb_read_status": (I, [P, SZ, P, ctypes.POINTER(I)]),
         "tb_decode_attn_noalloc": (I, [P, P, P, P, P, P, P]),
+        "tb_diag_exp2": (I, [P, P, ctypes.c_int64, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -302,6 +303,11 @@ def tb_decode_attn_noalloc(desc: DecodeDesc, q, Kc, Vc, lens, out, stream=None):
     Calls that overlap on the GPU race on that array."""
     _check(load().tb_decode_attn_noalloc(desc.ref(), _ptr(q), _ptr(Kc), _ptr(Vc), _ptr(lens), _ptr(out),
                                          _stream(stream)), "tb_decode_attn_noalloc")
+
+
+def tb_diag_exp2(x, y, stream=None):
+    """y = 2^x by the scoring kernels' FMA-pipe exponential (diagnostic)."""
+    _check(load().tb_diag_exp2(_ptr(x), _ptr(y), int(x.numel()), _stream(stream)), "tb_diag_exp2")
 
 
 def tb_read_status(workspace, workspace_bytes=None, stream=None):

@@ -1,24 +1,27 @@
-// Decode-step attention over the compacted bf16 cache, TMA-staged.
+// Decode-step attention over the compacted bf16 cache, TMA-staged, on
+// mma.sync tensor-core fragments.
 //
 // Same result as the portable kernel in k_decode.cu (one query per head,
 // softmax over the request's first len keys, attention definition of
 // "FLOPs-based Modeling"), organised for HBM bandwidth: each CTA takes one
 // (request, KV head, key split) and streams its K and V rows through a
 // 3-stage ring of 64-key tiles that one thread fills with 2-D TMA copies
-// (128-byte swizzle, so that reading a key row or a value column from shared
-// memory is free of bank conflicts). The G query heads of the group share
-// every tile, so each K/V byte is read from HBM once per decode step.
+// (128-byte swizzle, so ldmatrix reads are free of bank conflicts). The G
+// query heads of the group share every tile, so each K/V byte is read from
+// HBM once per decode step.
 //
-// Per 64-key tile (128 threads):
-//   scores   thread pair (2i, 2i+1) owns key i, each half of the head dim;
-//            q . k for the G heads in fp32, pair-combined with one shuffle;
-//   softmax  per-head tile max across the CTA, running max / rescale (log2
-//            domain), p = 2^(t - m) written to shared memory;
-//   p . V    thread t owns two dims of the output for all heads and half of
-//            the tile's keys; the halves are added at the end.
-// Partial (max, sum, unnormalised output) per split go to the workspace; the
-// CTA that finishes last among a (request, KV head)'s splits (a counter in
-// the workspace, zeroed by every call) merges them and writes the output.
+// Warp w owns keys [16w, 16w + 16) of every tile and keeps its own running
+// max / sum / output for the G heads (rows of a 16-row MMA tile; rows past G
+// are zero queries whose results are dropped):
+//   S = Q K^T      mma.m16n8k16 bf16 -> fp32, K fragments by ldmatrix;
+//   softmax        per row over the warp's keys, log2 domain, fp32;
+//   O += P V       P in fp32 is split into a bf16 part and a bf16 residual,
+//                  both multiplied by V (ldmatrix.trans) and accumulated in
+//                  fp32, so P enters with ~16 significant bits.
+// At the end the four warps merge in shared memory into the split's partial
+// (max, sum, unnormalised output); the CTA that finishes last among a
+// (request, KV head)'s splits (a counter in the workspace, zeroed by every
+// call) merges the splits and writes the output.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -34,18 +37,17 @@ constexpr int kTile = 64;
 constexpr int kStages = 3;
 constexpr int kBox = 64 * 128;  // 64 rows x 128 B
 
-template <int D, int G>
+template <int D>
 struct DGeo {
   static constexpr int KH = D / 64;
-  static constexpr int Gp = (G + 3) & ~3;
-  static constexpr int kStageBytes = 2 * KH * kBox;      // K and V halves of one tile
+  static constexpr int kStageBytes = 2 * KH * kBox;  // K and V halves of one tile
   static constexpr int kRing = kStages * kStageBytes;
-  static constexpr int kQOff = kRing;                    // q: G x D floats
-  static constexpr int kPOff = kQOff + G * D * 4;        // p: kTile x Gp floats
-  static constexpr int kRedOff = kPOff + kTile * Gp * 4; // reductions:
-  // per-warp head values (4 x G), then (KPARTS-1) x G x D output parts
-  static constexpr int kBarOff = (kRedOff + 4 * G * 4 + G * (256 - D) * 4 + 15) & ~15;
-  static constexpr int kSmem = kBarOff + 64 + 1024;      // + alignment slack
+  // after the key loop the ring holds the cross-warp merge: O, m, l per warp
+  static constexpr int kMergeO = 4 * 16 * D * 4;
+  static_assert(kMergeO + 4 * 16 * 8 <= kRing, "merge area must fit in the ring");
+  static constexpr int kMaxSplits = kRing / (16 * 4);  // weights table [G <= 16][splits]
+  static constexpr int kBarOff = kRing;
+  static constexpr int kSmem = kBarOff + 64 + 1024;  // + alignment slack
 };
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
@@ -58,15 +60,42 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
-__device__ __forceinline__ void bf16x8_to_f32(const uint4 v, float (&f)[8]) {
-  f[0] = __uint_as_float(v.x << 16);
-  f[1] = __uint_as_float(v.x & 0xffff0000u);
-  f[2] = __uint_as_float(v.y << 16);
-  f[3] = __uint_as_float(v.y & 0xffff0000u);
-  f[4] = __uint_as_float(v.z << 16);
-  f[5] = __uint_as_float(v.z & 0xffff0000u);
-  f[6] = __uint_as_float(v.w << 16);
-  f[7] = __uint_as_float(v.w & 0xffff0000u);
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+
+// c (16x8 fp32) += a (16x16 bf16, row) * b (16x8 bf16, col)
+__device__ __forceinline__ void mma_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                          uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// two fp32 -> bf16x2 (lo in the low half), round to nearest even
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+// byte offset of 16-byte chunk `chunk` (of the D/8 in a row) of tile row `row`
+// inside a stage half (K or V) laid out as KH boxes of 64 rows x 128 B, 128B-swizzled
+__device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
+  return (uint32_t)((chunk >> 3) * kBox + row * 128 + (((chunk & 7) ^ (row & 7)) << 4));
 }
 
 template <int D, int G>
@@ -76,19 +105,18 @@ __global__ void __launch_bounds__(kThreads, 2)
                const int32_t* __restrict__ lens, float* __restrict__ part_o,
                float2* __restrict__ part_ml, int32_t* __restrict__ counters,
                void* __restrict__ out, int32_t* __restrict__ status) {
-  using Gm = DGeo<D, G>;
+  using Gm = DGeo<D>;
+  constexpr int KS = D / 16;  // k-steps of Q K^T
+  constexpr int NT = D / 8;   // n-tiles of P V
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  float* qs = reinterpret_cast<float*>(smem + Gm::kQOff);    // [G][D]
-  float* ps = reinterpret_cast<float*>(smem + Gm::kPOff);    // [kTile][Gp]
-  float* red = reinterpret_cast<float*>(smem + Gm::kRedOff); // [4 warps][G], then o halves
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + Gm::kBarOff);
   int* abort_flag = reinterpret_cast<int*>(smem + Gm::kBarOff + 8 * kStages);
   int* last_flag = abort_flag + 1;
-  constexpr int Gp = Gm::Gp;
 
   const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int r0 = lane >> 2, qd = lane & 3;  // fragment row (and row + 8), column pair
   int len = lens[b];
   {
     const int64_t cap64 = p.max_len < (int64_t)p.cache_cap[b] ? p.max_len : (int64_t)p.cache_cap[b];
@@ -100,8 +128,8 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   const int k0 = split * p.split_len;
   const int k1 = min(len, k0 + p.split_len);
-  const size_t part_base = ((size_t)b * p.hq + (size_t)g * G) * p.splits + split;
   const int ntiles = k1 > k0 ? (k1 - k0 + kTile - 1) / kTile : 0;
+  const size_t part_base = ((size_t)b * p.hq + (size_t)g * G) * p.splits + split;
   const int row0 = (int)((int64_t)g * p.cache_rows + p.cache_off[b]) + k0;
 
   if (tid == 0) {
@@ -110,8 +138,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     *last_flag = 0;
     tc::fence_barrier_init();
   }
-  const uint16_t* qg = q + ((size_t)b * p.hq + (size_t)g * G) * D;
-  for (int e = tid; e < G * D; e += kThreads) qs[e] = __uint_as_float((uint32_t)qg[e] << 16);
   __syncthreads();
 
   auto issue = [&](int t) {
@@ -130,22 +156,26 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (; issued < kStages && issued < ntiles; ++issued) issue(issued);
   }
 
-  const float c = p.scale_log2;
-  // score role: key kk = tid / 2, half hh = tid % 2 of the head dim
-  const int kk = tid >> 1, hh = tid & 1;
-  // p.V role: dim pair dp (dims 2dp, 2dp+1), key half kh
-  constexpr int DP = D / 2;                 // dim pairs
-  constexpr int KPARTS = kThreads / DP;     // 2 for d=128, 4 for d=64
-  constexpr int KPER = kTile / KPARTS;
-  const int dp = tid % DP, kh = tid / DP;
-  float m_run[G], l_run[G], o0[G], o1[G];
+  // Q fragments (rows >= G are zero queries)
+  uint32_t aq[KS][4];
+  {
+    const uint32_t* qg = reinterpret_cast<const uint32_t*>(q + ((size_t)b * p.hq + (size_t)g * G) * D);
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-    m_run[h] = -INFINITY;
-    l_run[h] = 0.f;
-    o0[h] = 0.f;
-    o1[h] = 0.f;
+    for (int kk = 0; kk < KS; ++kk) {
+      const int w0 = (kk * 16 + 2 * qd) >> 1;  // bf16 pair index in a row
+      aq[kk][0] = r0 < G ? qg[r0 * (D / 2) + w0] : 0u;
+      aq[kk][1] = r0 + 8 < G ? qg[(r0 + 8) * (D / 2) + w0] : 0u;
+      aq[kk][2] = r0 < G ? qg[r0 * (D / 2) + w0 + 4] : 0u;
+      aq[kk][3] = r0 + 8 < G ? qg[(r0 + 8) * (D / 2) + w0 + 4] : 0u;
+    }
   }
+
+  const float c = p.scale_log2;
+  float o[NT][4];
+#pragma unroll
+  for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  const int kb = warp * 16;  // this warp's first key in a tile
   bool ok = true;
 
   for (int t = 0; t < ntiles; ++t) {
@@ -155,155 +185,163 @@ __global__ void __launch_bounds__(kThreads, 2)
       ok = false;
       break;
     }
-    const uint8_t* kst = smem + s * Gm::kStageBytes;
-    const uint8_t* vst = kst + Gm::KH * kBox;
+    const uint32_t kst = tc::smem_addr(smem + s * Gm::kStageBytes);
+    const uint32_t vst = kst + (uint32_t)(Gm::KH * kBox);
     const int nvalid = min(kTile, k1 - (k0 + t * kTile));
-
-    // ---- scores for key kk, dims of half hh
-    float dot[G];
+    if (kb < nvalid) {
+      // rows past len may hold anything (even NaN): clear this warp's V rows there
+      if (kb + 16 > nvalid) {
+        uint8_t* vrow = smem + s * Gm::kStageBytes + Gm::KH * kBox;
+        for (int e = lane; e < (kb + 16 - nvalid) * (D / 8); e += 32) {
+          const int row = nvalid + e / (D / 8), chunk = e % (D / 8);
+          *reinterpret_cast<uint4*>(vrow + sw_off(row, chunk)) = make_uint4(0, 0, 0, 0);
+        }
+        __syncwarp();
+      }
+      // ---- S = Q K^T over this warp's 16 keys
+      float sc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+      {
+        const int krow = kb + (lane & 7) + ((lane >> 4) << 3);
+        const int ksel = (lane >> 3) & 1;
 #pragma unroll
-    for (int h = 0; h < G; ++h) dot[h] = 0.f;
-    constexpr int CH = D / 16;  // 16-byte chunks per half row
+        for (int kk = 0; kk < KS; ++kk) {
+          uint32_t bk[4];
+          ldsm_x4(kst + sw_off(krow, 2 * kk + ksel), bk);
+          mma_16816(sc[0], aq[kk], bk[0], bk[1]);
+          mma_16816(sc[1], aq[kk], bk[2], bk[3]);
+        }
+      }
+      // ---- online softmax per row (r0: elements 0,1; r0 + 8: elements 2,3)
+      float corr[2];
 #pragma unroll
-    for (int c8 = 0; c8 < CH; ++c8) {
-      // the two halves start at different 16-byte chunks: no shared bank
-      const int cc = D == 128 ? ((c8 + 4 * hh) & 7) : c8;
-      const int dim0 = hh * (D / 2) + cc * 8;
-      const int box = dim0 >> 6, chunk = (dim0 & 63) >> 3;
-      const uint4 raw = *reinterpret_cast<const uint4*>(kst + box * kBox + kk * 128 +
-                                                        ((chunk ^ (kk & 7)) << 4));
-      float kf[8];
-      bf16x8_to_f32(raw, kf);
+      for (int hr = 0; hr < 2; ++hr) {
+        float mx = -INFINITY;
 #pragma unroll
-      for (int h = 0; h < G; ++h) {
-        const float4 qa = *reinterpret_cast<const float4*>(qs + h * D + dim0);
-        const float4 qb = *reinterpret_cast<const float4*>(qs + h * D + dim0 + 4);
-        float a = dot[h];
-        a = fmaf(qa.x, kf[0], a);
-        a = fmaf(qa.y, kf[1], a);
-        a = fmaf(qa.z, kf[2], a);
-        a = fmaf(qa.w, kf[3], a);
-        a = fmaf(qb.x, kf[4], a);
-        a = fmaf(qb.y, kf[5], a);
-        a = fmaf(qb.z, kf[6], a);
-        a = fmaf(qb.w, kf[7], a);
-        dot[h] = a;
+        for (int n = 0; n < 2; ++n)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            const int key = kb + n * 8 + 2 * qd + j;
+            const float x = key < nvalid ? sc[n][2 * hr + j] * c : -INFINITY;
+            sc[n][2 * hr + j] = x;
+            mx = fmaxf(mx, x);
+          }
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        const float m_new = fmaxf(m_run[hr], mx);  // finite: key kb is valid
+        corr[hr] = fast_exp2(m_run[hr] - m_new);
+        m_run[hr] = m_new;
+        float ls = 0.f;
+#pragma unroll
+        for (int n = 0; n < 2; ++n)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            const float pv = fast_exp2(sc[n][2 * hr + j] - m_new);
+            sc[n][2 * hr + j] = pv;
+            ls += pv;
+          }
+        l_run[hr] = l_run[hr] * corr[hr] + ls;
+      }
+      if (__any_sync(0xffffffffu, corr[0] != 1.f || corr[1] != 1.f)) {
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+          o[n][0] *= corr[0];
+          o[n][1] *= corr[0];
+          o[n][2] *= corr[1];
+          o[n][3] *= corr[1];
+        }
+      }
+      // ---- P as bf16 value + bf16 residual (A fragments, keys along k)
+      uint32_t ph[4], pl[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int n = i >> 1, e0 = (i & 1) * 2;
+        const float x0 = sc[n][e0], x1 = sc[n][e0 + 1];
+        ph[i] = pack_bf16(x0, x1);
+        pl[i] = pack_bf16(x0 - bf16_lo(ph[i]), x1 - bf16_hi(ph[i]));
+      }
+      // A fragment order: a0 (row r0, keys 0-7), a1 (row r0+8, keys 0-7),
+      // a2 (row r0, keys 8-15), a3 (row r0+8, keys 8-15)
+      const uint32_t ah[4] = {ph[0], ph[1], ph[2], ph[3]};
+      const uint32_t al[4] = {pl[0], pl[1], pl[2], pl[3]};
+      // ---- O += P V
+      {
+        const int vrow = kb + (lane & 7) + (((lane >> 3) & 1) << 3);
+        const int vsel = lane >> 4;
+#pragma unroll
+        for (int jj = 0; jj < NT / 2; ++jj) {
+          uint32_t bv[4];
+          ldsm_x4_t(vst + sw_off(vrow, 2 * jj + vsel), bv);
+          mma_16816(o[2 * jj], ah, bv[0], bv[1]);
+          mma_16816(o[2 * jj], al, bv[0], bv[1]);
+          mma_16816(o[2 * jj + 1], ah, bv[2], bv[3]);
+          mma_16816(o[2 * jj + 1], al, bv[2], bv[3]);
+        }
       }
     }
-    float tmax[G];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      dot[h] += __shfl_xor_sync(0xffffffffu, dot[h], 1);
-      dot[h] = kk < nvalid ? dot[h] * c : -INFINITY;
-      float m = dot[h];
-      for (int off = 2; off < 32; off <<= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-      tmax[h] = m;
-    }
-    if (lane == 0)
-#pragma unroll
-      for (int h = 0; h < G; ++h) red[warp * G + h] = tmax[h];
-    __syncthreads();
-    float corr[G];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      const float m_tile = fmaxf(fmaxf(red[h], red[G + h]), fmaxf(red[2 * G + h], red[3 * G + h]));
-      const float m_new = fmaxf(m_run[h], m_tile);
-      corr[h] = fast_exp2(m_run[h] - m_new);
-      m_run[h] = m_new;
-      const float pv = fast_exp2(dot[h] - m_new);
-      l_run[h] = l_run[h] * corr[h] + (hh == 0 ? pv : 0.f);
-      if (hh == 0) ps[kk * Gp + h] = pv;
-    }
-    __syncthreads();
-
-    // ---- p . V for dims (2dp, 2dp+1), keys kh*KPER .. +KPER
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      o0[h] *= corr[h];
-      o1[h] *= corr[h];
-    }
-    const int vbox = (2 * dp) >> 6, vchunk = ((2 * dp) & 63) >> 3, vin = ((2 * dp) & 7) * 2;
-#pragma unroll 4
-    for (int j = 0; j < KPER; ++j) {
-      const int key = kh * KPER + j;
-      if (key >= nvalid) break;  // rows past len may hold anything (even NaN)
-      const uint32_t v2 = *reinterpret_cast<const uint32_t*>(
-          vst + vbox * kBox + key * 128 + ((vchunk ^ (key & 7)) << 4) + vin);
-      const float va = __uint_as_float(v2 << 16), vb = __uint_as_float(v2 & 0xffff0000u);
-      const float* pk = ps + key * Gp;
-#pragma unroll
-      for (int h = 0; h < G; ++h) {
-        const float pw = pk[h];
-        o0[h] = fmaf(pw, va, o0[h]);
-        o1[h] = fmaf(pw, vb, o1[h]);
-      }
-    }
-    __syncthreads();  // stage s and ps are free again
+    __syncthreads();  // stage s is free again
     if (tid == 0 && issued < ntiles) {
       issue(issued);
       ++issued;
     }
   }
 
-  if (ok && ntiles > 0) {
-    // add the key parts of the output, reduce l over the CTA
-    float* ored = red + 4 * G;  // [KPARTS-1][G][D]
-    if (kh > 0) {
-#pragma unroll
-      for (int h = 0; h < G; ++h) {
-        ored[((kh - 1) * G + h) * D + 2 * dp] = o0[h];
-        ored[((kh - 1) * G + h) * D + 2 * dp + 1] = o1[h];
+  if (!ok) {
+    if (tid == 0) {
+      // drain the copies still in flight before the CTA exits
+      int dummy = 0;
+      for (int s = 0; s < kStages && s < issued; ++s) {
+        const int last = issued - 1 - ((issued - 1 - s) % kStages);
+        tc::mbar_wait(&full[s], (uint32_t)((last / kStages) & 1), &dummy, status);
       }
     }
-    float lsum[G];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      float v = l_run[h];
-      for (int off = 1; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      lsum[h] = v;
-    }
-    __syncthreads();
-    if (lane == 0)
-#pragma unroll
-      for (int h = 0; h < G; ++h) red[warp * G + h] = lsum[h];
-    __syncthreads();
-    if (kh == 0) {
-#pragma unroll
-      for (int h = 0; h < G; ++h) {
-        float a = o0[h], bb = o1[h];
-        for (int q2 = 1; q2 < KPARTS; ++q2) {
-          a += ored[((q2 - 1) * G + h) * D + 2 * dp];
-          bb += ored[((q2 - 1) * G + h) * D + 2 * dp + 1];
-        }
-        float* po = part_o + (part_base + (size_t)h * p.splits) * D;
-        po[2 * dp] = a;
-        po[2 * dp + 1] = bb;
-      }
-    }
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      if (tid == h) {
-        const float l = red[h] + red[G + h] + red[2 * G + h] + red[3 * G + h];
-        part_ml[part_base + (size_t)h * p.splits] = make_float2(m_run[h], l);
-      }
-    }
-  } else if (ok) {  // an empty split: neutral partials
-    for (int e = tid; e < G * D; e += kThreads) {
-      const int h = e / D, dim = e % D;
-      part_o[(part_base + (size_t)h * p.splits) * D + dim] = 0.f;
-      if (dim == 0) part_ml[part_base + (size_t)h * p.splits] = make_float2(-INFINITY, 0.f);
-    }
-  } else if (tid == 0) {
-    // drain the copies still in flight before the CTA exits
-    int dummy = 0;
-    for (int s = 0; s < kStages && s < issued; ++s) {
-      const int last = issued - 1 - ((issued - 1 - s) % kStages);
-      tc::mbar_wait(&full[s], (uint32_t)((last / kStages) & 1), &dummy, status);
-    }
+    return;
   }
-  if (!ok) return;
 
-  // the last split CTA of this (request, KV head) merges every split
+  // ---- merge the four warps: O, m, l through shared memory (the ring is free)
+#pragma unroll
+  for (int hr = 0; hr < 2; ++hr) {
+    l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 1);
+    l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 2);
+  }
+  float* mo = reinterpret_cast<float*>(smem);                // [4][16][D]
+  float* mml = reinterpret_cast<float*>(smem + Gm::kMergeO);  // [4][16][2]
+#pragma unroll
+  for (int n = 0; n < NT; ++n) {
+    const int dim = n * 8 + 2 * qd;
+    mo[(warp * 16 + r0) * D + dim] = o[n][0];
+    mo[(warp * 16 + r0) * D + dim + 1] = o[n][1];
+    mo[(warp * 16 + r0 + 8) * D + dim] = o[n][2];
+    mo[(warp * 16 + r0 + 8) * D + dim + 1] = o[n][3];
+  }
+  if (qd == 0) {
+    mml[(warp * 16 + r0) * 2] = m_run[0];
+    mml[(warp * 16 + r0) * 2 + 1] = l_run[0];
+    mml[(warp * 16 + r0 + 8) * 2] = m_run[1];
+    mml[(warp * 16 + r0 + 8) * 2 + 1] = l_run[1];
+  }
+  __syncthreads();
+  for (int e = tid; e < G * D; e += kThreads) {
+    const int h = e / D, dim = e % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, mml[(w * 16 + h) * 2]);
+    float L = 0.f, O = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float mw = mml[(w * 16 + h) * 2];
+        if (mw != -INFINITY) {
+          const float wt = fast_exp2(mw - M);
+          L = fmaf(mml[(w * 16 + h) * 2 + 1], wt, L);
+          O = fmaf(mo[(w * 16 + h) * D + dim], wt, O);
+        }
+      }
+    }
+    part_o[(part_base + (size_t)h * p.splits) * D + dim] = O;
+    if (dim == 0) part_ml[part_base + (size_t)h * p.splits] = make_float2(M, L);
+  }
+
+  // ---- the last split CTA of this (request, KV head) merges every split
   __threadfence();
   __syncthreads();
   if (tid == 0) *last_flag = atomicAdd(&counters[b * p.hkv + g], 1) == p.splits - 1;
@@ -311,28 +349,51 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (!*last_flag) return;
   __threadfence();
   const size_t head0 = ((size_t)b * p.hq + (size_t)g * G) * p.splits;
-  for (int e = tid; e < G * D; e += kThreads) {
-    const int h = e / D, dim = e % D;
+  // per head: weight of split s = 2^(m_s - M) / L, lanes over splits
+  float* wts = reinterpret_cast<float*>(smem);  // [G][splits] (the ring is free)
+  for (int h = warp; h < G; h += kThreads / 32) {
     const size_t hb = head0 + (size_t)h * p.splits;
-    float m = -INFINITY;
-    for (int sp = 0; sp < p.splits; ++sp) m = fmaxf(m, __ldcg(&part_ml[hb + sp]).x);
-    float l = 0.f, o = 0.f;
-    if (m != -INFINITY) {
-      for (int sp = 0; sp < p.splits; ++sp) {
-        const float2 ml = __ldcg(&part_ml[hb + sp]);
-        if (ml.y > 0.f) {
-          const float wgt = fast_exp2(ml.x - m);
-          l = fmaf(ml.y, wgt, l);
-          o = fmaf(__ldcg(&part_o[(hb + sp) * D + dim]), wgt, o);
-        }
-      }
+    float M = -INFINITY;
+    for (int sp = lane; sp < p.splits; sp += 32) M = fmaxf(M, __ldcg(&part_ml[hb + sp]).x);
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float L = 0.f;
+    for (int sp = lane; sp < p.splits; sp += 32) {
+      const float2 ml = __ldcg(&part_ml[hb + sp]);
+      const float wgt = (M != -INFINITY && ml.y > 0.f) ? fast_exp2(ml.x - M) : 0.f;
+      wts[h * p.splits + sp] = wgt;
+      L = fmaf(ml.y, wgt, L);
     }
-    const float r = l > 0.f ? o / l : 0.f;
-    const size_t oi = ((size_t)b * p.hq + (size_t)g * G + h) * D + dim;
+    for (int off = 16; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    __syncwarp();
+    for (int sp = lane; sp < p.splits; sp += 32) wts[h * p.splits + sp] *= inv;
+  }
+  __syncthreads();
+  // outputs in float4 groups of dims; every split's partial is an independent load
+  constexpr int D4 = D / 4;
+  for (int e = tid; e < G * D4; e += kThreads) {
+    const int h = e / D4, d4 = e % D4;
+    const size_t hb = head0 + (size_t)h * p.splits;
+    const float* wh = wts + h * p.splits;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+    for (int sp = 0; sp < p.splits; ++sp) {
+      const float wgt = wh[sp];
+      const float4 ov = __ldcg(reinterpret_cast<const float4*>(part_o + (hb + sp) * D) + d4);
+      acc.x = fmaf(ov.x, wgt, acc.x);
+      acc.y = fmaf(ov.y, wgt, acc.y);
+      acc.z = fmaf(ov.z, wgt, acc.z);
+      acc.w = fmaf(ov.w, wgt, acc.w);
+    }
+    const size_t oi = ((size_t)b * p.hq + (size_t)g * G + h) * D + 4 * d4;
     if (p.out_dtype == TB_F32) {
-      static_cast<float*>(out)[oi] = r;
+      *reinterpret_cast<float4*>(static_cast<float*>(out) + oi) = acc;
     } else {
-      static_cast<uint16_t*>(out)[oi] = float_to_bf16_rne(r);
+      uint16_t* ob = static_cast<uint16_t*>(out) + oi;
+      ob[0] = float_to_bf16_rne(acc.x);
+      ob[1] = float_to_bf16_rne(acc.y);
+      ob[2] = float_to_bf16_rne(acc.z);
+      ob[3] = float_to_bf16_rne(acc.w);
     }
   }
 }
@@ -341,7 +402,7 @@ template <int D, int G>
 cudaError_t launch_g(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
                      const void* q, const int32_t* lens, float* part_o, float2* part_ml,
                      int32_t* counters, void* out, int32_t* status, cudaStream_t s) {
-  using Gm = DGeo<D, G>;
+  using Gm = DGeo<D>;
   auto kern = decode_tma<D, G>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
@@ -370,8 +431,9 @@ cudaError_t launch_d(const DecodeParams& p, const CUtensorMap& tk, const CUtenso
 
 bool decode_tma_supported(const DecodeParams& p) {
   const int g = p.group;
-  const bool g_ok = (g >= 1 && g <= 8) || g == 12 || g == 16;
-  return p.dtype == TB_BF16 && (p.d == 64 || p.d == 128) && g_ok &&
+  const bool g_ok = (g >= 1 && g <= 8) || g == 12 || g == 16;  // rows of one 16-row MMA tile
+  const int max_splits = p.d == 64 ? DGeo<64>::kMaxSplits : DGeo<128>::kMaxSplits;
+  return p.dtype == TB_BF16 && (p.d == 64 || p.d == 128) && g_ok && p.splits <= max_splits &&
          (uint64_t)p.hkv * (uint64_t)p.cache_rows < (1ull << 31);
 }
 

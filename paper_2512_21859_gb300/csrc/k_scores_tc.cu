@@ -17,9 +17,11 @@
 //                        the key tiles in reverse order so that the tail the
 //                        first pass loaded last is still in L2.
 //
-// Warp roles (384 threads, one CTA per SM): warp 0 issues TMA loads, warp 1
+// Warp roles (640 threads, one CTA per SM): warp 0 issues TMA loads, warp 1
 // issues the MMAs (one elected thread), warp 2 owns the TMEM allocation, and
-// warps 4..11 (two warpgroups) are the epilogue. Shared memory holds the
+// warps 4..19 are the epilogue: four per TMEM lane quadrant, each taking a
+// quarter of the accumulator columns (the epilogue is latency-bound, so it
+// wants many warps). Shared memory holds the
 // window rows once and a 4-stage ring of key tiles; TMEM holds two 256-column
 // accumulators so the MMA of tile t+1 overlaps the epilogue of tile t.
 #include <cuda.h>
@@ -37,11 +39,16 @@ namespace {
 
 constexpr int kTileKeys = 128;
 constexpr int kStages = 4;
-constexpr int kThreads = 384;
+constexpr int kThreads = 640;
 constexpr int kEpiWarp0 = 4;
-constexpr int kEpiWarps = 8;
+constexpr int kEpiWarps = 16;  // four per TMEM lane quadrant, each on a quarter of the columns
 constexpr uint32_t kTmemCols = 512;
 constexpr int kBoxBytes = 128 * 128;  // one TMA box: 128 rows x 64 bf16
+// Of every 32 exponentials an epilogue thread takes, the first kMufuElems go
+// to the MUFU unit and the rest to the FMA pipes (tc::exp2_poly2). Measured on
+// GB300: sending 12 of 32 to the FMA pipes slowed both passes (the epilogue is
+// bound by latency, not by MUFU throughput), so all of them use MUFU.
+constexpr int kMufuElems = 32;
 
 template <int D>
 struct Geo {
@@ -53,8 +60,9 @@ struct Geo {
   static constexpr int kRingOff = kQBytes;
   static constexpr int kBarOff = kRingOff + kStages * kTileBytes;
   static constexpr int kCrOff = kBarOff + 1024;
-  static constexpr int kXOff = kCrOff + 256 * 4;
-  static constexpr int kSmem = kXOff + 2 * 128 * 4 + 1024;  // + alignment slack
+  static constexpr int kXOff = kCrOff + 256 * 4;       // pass 2: 2 x 3 x 128 partial sums
+  static constexpr int kMOff = kXOff + 2 * 3 * 128 * 4;  // pass 1: 256 (max, sum) pairs
+  static constexpr int kSmem = kMOff + 256 * 8 + 1024;   // + alignment slack
 };
 
 struct Bars {
@@ -111,8 +119,8 @@ __device__ __forceinline__ uint32_t setup(Bars* bars) {
     }
     tc::mbar_init(&bars->qfull, 1);
     for (int x = 0; x < 2; ++x) {
-      tc::mbar_init(&bars->xfull[x], kEpiWarps / 2);
-      tc::mbar_init(&bars->xempty[x], kEpiWarps / 2);
+      tc::mbar_init(&bars->xfull[x], kEpiWarps * 3 / 4);
+      tc::mbar_init(&bars->xempty[x], kEpiWarps / 4);
     }
     bars->abort = 0;
     tc::fence_barrier_init();
@@ -167,6 +175,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* q_s = smem;
   uint8_t* ring = smem + G::kRingOff;
   Bars* bars = reinterpret_cast<Bars*>(smem + G::kBarOff);
+  float2* mrg = reinterpret_cast<float2*>(smem + G::kMOff);
+  bool my_ok = false;
+  float my_m = -INFINITY, my_l = 0.f;
 
   const int item = blockIdx.x;
   const ItemInfo info = locate(p, item, false);
@@ -226,7 +237,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp >= kEpiWarp0) {
-    const int e = warp - kEpiWarp0, wg = e >> 2, quad = warp & 3;
+    // rows: row block wg, TMEM lane quadrant quad; columns: half `half` of the tile
+    const int e = warp - kEpiWarp0, sub = e >> 2, quad = warp & 3;
+    const int wg = sub >> 1, half = sub & 1;
     const int row = wg * 128 + quad * 32 + lane;
     const int w = row % p.window;
     const int vis_end = min(rq.n, rq.p + w + 1);  // keys [0, vis_end) visible to the row
@@ -246,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int key0 = info.j0 + it * kTileKeys;
         const bool all_vis = key0 + kTileKeys <= rq.p;
 #pragma unroll 1
-        for (int ch = 0; ch < 4; ++ch) {
+        for (int ch = 2 * half; ch < 2 * half + 2; ++ch) {
           float v[32];
           __syncwarp();
           tc::tmem_ld32(taddr + ch * 32, v);
@@ -256,9 +269,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 32; ++i)
               if (key0 + ch * 32 + i >= vis_end) v[i] = -INFINITY;
           }
-          float mx = v[0];
+          // chunk max with three-input max (tree of 16 + 5 + 2 + 1 ops)
+          float mt[11];
 #pragma unroll
-          for (int i = 1; i < 32; ++i) mx = fmaxf(mx, v[i]);
+          for (int i = 0; i < 10; ++i) mt[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+          mt[10] = fmaxf(v[30], v[31]);
+          const float mx = tc::max3(tc::max3(mt[0], mt[1], mt[2]), tc::max3(mt[3], mt[4], mt[5]),
+                                    tc::max3(tc::max3(mt[6], mt[7], mt[8]), mt[9], mt[10]));
           const float m_new = fmaxf(m_run, mx * c);
           if (m_new != -INFINITY) {  // some key of this chunk is visible
             if (m_new > m_run) {
@@ -267,15 +284,26 @@ __global__ void __launch_bounds__(kThreads, 1)
               l_comp *= sc;
               m_run = m_new;
             }
-            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+            // 2^(v c - m) in packed pairs, summed in two packed accumulators
+            const uint64_t cc = tc::pk2(c, c), mm = tc::pk2(-m_run, -m_run);
+            uint64_t acc0 = 0, acc1 = 0;
 #pragma unroll
             for (int i = 0; i < 32; i += 4) {
-              s0 += fast_exp2(fmaf(v[i], c, -m_run));
-              s1 += fast_exp2(fmaf(v[i + 1], c, -m_run));
-              s2 += fast_exp2(fmaf(v[i + 2], c, -m_run));
-              s3 += fast_exp2(fmaf(v[i + 3], c, -m_run));
+              const float2 a = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), cc, mm));
+              const float2 bq = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), cc, mm));
+              float2 ea, eb;
+              if (i < kMufuElems) {
+                ea = make_float2(fast_exp2(a.x), fast_exp2(a.y));
+                eb = make_float2(fast_exp2(bq.x), fast_exp2(bq.y));
+              } else {
+                ea = tc::exp2_poly2(a.x, a.y);
+                eb = tc::exp2_poly2(bq.x, bq.y);
+              }
+              acc0 = tc::add2(acc0, tc::pk2(ea.x, ea.y));
+              acc1 = tc::add2(acc1, tc::pk2(eb.x, eb.y));
             }
-            const float term = ((s0 + s1) + (s2 + s3)) - l_comp;
+            const float2 s01 = tc::upk2(tc::add2(acc0, acc1));
+            const float term = (s01.x + s01.y) - l_comp;
             const float tsum = l_run + term;
             l_comp = (tsum - l_run) - term;
             l_run = tsum;
@@ -286,7 +314,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
     }
-    if (ok && wg < RB && row < M) partial[(size_t)item * M + row] = make_float2(m_run, l_run);
+    // the second column half hands its (max, sum) to the first
+    if (half == 1) mrg[row] = make_float2(ok ? m_run : NAN, l_run);
+    my_ok = ok;
+    my_m = m_run;
+    my_l = l_run;
+  }
+  __syncthreads();
+  if (warp >= kEpiWarp0) {
+    const int e = warp - kEpiWarp0, sub = e >> 2, quad = warp & 3;
+    const int wg = sub >> 1, half = sub & 1;
+    const int row = wg * 128 + quad * 32 + lane;
+    if (half == 0 && wg < RB && row < M) {
+      const float2 o = mrg[row];
+      if (my_ok && !isnan(o.x)) {
+        const float m = fmaxf(my_m, o.x);
+        const float l = (m == -INFINITY) ? 0.f
+                                        : my_l * fast_exp2(my_m - m) + o.y * fast_exp2(o.x - m);
+        partial[(size_t)item * M + row] = make_float2(m, l);
+      }
+    }
   }
   teardown(bars, tmem, issued, committed, status);
 }
@@ -319,7 +366,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
   const float* rc = rowc + ((size_t)info.b * p.hkv + info.g) * M;
-  for (int r = threadIdx.x; r < 256; r += blockDim.x) cr[r] = r < M ? rc[r] : INFINITY;
+  float* ncr = cr;  // -c_row; -inf for padding rows so that their terms vanish
+  for (int r = threadIdx.x; r < 256; r += blockDim.x) ncr[r] = r < M ? -rc[r] : -INFINITY;
   const uint32_t tmem = setup(bars);
   volatile int* abort = &bars->abort;
   int issued = 0, committed = 0;
@@ -368,7 +416,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp >= kEpiWarp0) {
-    const int e = warp - kEpiWarp0, wg = e >> 2, quad = warp & 3;
+    // keys: TMEM lane quadrant quad; window rows (columns): quarter `sub`
+    const int e = warp - kEpiWarp0, sub = e >> 2, quad = warp & 3;
     const int key = quad * 32 + lane;  // TMEM lane = key within the tile
     const float c = p.scale_log2;
     float* out = scores + (size_t)info.g * p.score_rows + rq.score_off;
@@ -380,40 +429,52 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(a * 256);
       float acc = 0.f;
 #pragma unroll 1
-      for (int ch = 0; ch < 4; ++ch) {
-        const int c0 = wg * 128 + ch * 32;
+      for (int ch = 0; ch < 2; ++ch) {
+        const int c0 = sub * 64 + ch * 32;
         if (c0 >= NP) break;
         float v[32];
         __syncwarp();
         tc::tmem_ld32(taddr + c0, v);
         tc::tmem_ld_wait();
-        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+        // 2^(v c - c_row) in packed pairs; -c_row pairs come from shared memory
+        const uint64_t c2 = tc::pk2(c, c);
+        uint64_t a0 = 0, a1 = 0;
 #pragma unroll
         for (int i = 0; i < 32; i += 4) {
-          const float4 cc = *reinterpret_cast<const float4*>(cr + c0 + i);
-          s0 += fast_exp2(fmaf(v[i], c, -cc.x));
-          s1 += fast_exp2(fmaf(v[i + 1], c, -cc.y));
-          s2 += fast_exp2(fmaf(v[i + 2], c, -cc.z));
-          s3 += fast_exp2(fmaf(v[i + 3], c, -cc.w));
+          const float4 nc = *reinterpret_cast<const float4*>(ncr + c0 + i);
+          const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), c2, tc::pk2(nc.x, nc.y)));
+          const float2 y = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), c2, tc::pk2(nc.z, nc.w)));
+          float2 ex, ey;
+          if (i < kMufuElems) {
+            ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+            ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
+          } else {
+            ex = tc::exp2_poly2(x.x, x.y);
+            ey = tc::exp2_poly2(y.x, y.y);
+          }
+          a0 = tc::add2(a0, tc::pk2(ex.x, ex.y));
+          a1 = tc::add2(a1, tc::pk2(ey.x, ey.y));
         }
-        acc += (s0 + s1) + (s2 + s3);
+        const float2 s01 = tc::upk2(tc::add2(a0, a1));
+        acc += s01.x + s01.y;
       }
       tc::tc_fence_before();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
-      // combine the two warpgroups' halves of the window rows through a
-      // double-buffered hand-off (bounded mbarrier waits, no named barrier)
+      // combine the four quarters of the window rows through a double-buffered
+      // hand-off (bounded mbarrier waits, no named barrier); fixed sum order
       const int x = it & 1;
       const uint32_t xph = (uint32_t)((it >> 1) & 1);
-      if (wg == 1) {
+      if (sub > 0) {
         if (!tc::mbar_wait(&bars->xempty[x], xph ^ 1, abort, status)) break;
-        xbuf[x * 128 + key] = acc;
+        xbuf[(x * 3 + sub - 1) * 128 + key] = acc;
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&bars->xfull[x]);
       } else {
         if (!tc::mbar_wait(&bars->xfull[x], xph, abort, status)) break;
         const int j = info.j0 + t * kTileKeys + key;
-        if (j < info.j1) out[j] = acc + xbuf[x * 128 + key];
+        const float* xb = xbuf + x * 3 * 128;
+        if (j < info.j1) out[j] = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&bars->xempty[x]);
       }

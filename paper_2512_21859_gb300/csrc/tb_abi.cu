@@ -177,9 +177,9 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
     p->cache_off[b] = d->cache_offset[b];
     p->cache_cap[b] = (int32_t)d->cache_cap[b];
   }
-  // Split the keys so that about two CTAs per SM of a 152-SM part run, in
-  // whole 64-key tiles.
-  const int64_t target = 2 * 152;
+  // Split the keys so that about one CTA per SM of a 152-SM part runs, in
+  // whole 64-key tiles (each CTA keeps three tiles in flight).
+  const int64_t target = 152;
   const int64_t units = (int64_t)d->batch * d->hkv;
   int64_t splits = (target + units - 1) / units;
   const int64_t max_splits = (d->max_len + 63) / 64;

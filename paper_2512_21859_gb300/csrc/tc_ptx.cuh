@@ -179,8 +179,65 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
          | ((uint32_t)(m >> 4) << 24);  // M / 16
 }
 
-__device__ __forceinline__ void named_bar_sync(int id, int threads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+// ---------------------------------------------------------------------------
+// packed fp32 pairs (one instruction for two lanes of arithmetic)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t pk2(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ float2 upk2(uint64_t v) {
+  float2 r;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+  return r;
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t sub2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// 2^x for a pair of x <= ~0.5 on the FMA pipes instead of the MUFU unit (which
+// issues 16 exponentials per SM per clock). Cody-Waite split x = n + f with n
+// = round(x) (by adding 1.5 * 2^23) and f in [-0.5, 0.5]; 2^f by a degree-5
+// polynomial fitted for minimum relative error (exp2_poly_fit.py: 2.1e-7 in
+// fp32); 2^n added to the exponent field. x is clamped at -125 so that the
+// result stays a normal float; 2^-125 is far below anything that matters here.
+__device__ __forceinline__ float2 exp2_poly2(float x0, float x1) {
+  x0 = fmaxf(x0, -125.f);
+  x1 = fmaxf(x1, -125.f);
+  const uint64_t x = pk2(x0, x1);
+  const uint64_t magic = pk2(12582912.f, 12582912.f);  // 1.5 * 2^23
+  const uint64_t r = add2(x, magic);
+  const uint64_t f = sub2(x, sub2(r, magic));
+  uint64_t p = fma2(pk2(1.327647245e-03f, 1.327647245e-03f), f,
+                    pk2(9.675540961e-03f, 9.675540961e-03f));
+  p = fma2(p, f, pk2(5.550713092e-02f, 5.550713092e-02f));
+  p = fma2(p, f, pk2(2.402212024e-01f, 2.402212024e-01f));
+  p = fma2(p, f, pk2(6.931469440e-01f, 6.931469440e-01f));
+  p = fma2(p, f, pk2(1.000000119e+00f, 1.000000119e+00f));
+  const float2 pf = upk2(p), rf = upk2(r);
+  // low bits of r hold n (+ the magic's zero low bits): n << 23 shifts them into
+  // the exponent field, the magic's own bits shift out
+  return make_float2(__uint_as_float(__float_as_uint(pf.x) + (__float_as_uint(rf.x) << 23)),
+                     __uint_as_float(__float_as_uint(pf.y) + (__float_as_uint(rf.y) << 23)));
+}
+
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
 }  // namespace tc

@@ -351,3 +351,18 @@ def test_window_scores_stage():
     for b in range(2):
         s0, _, P, _ = request_slices(desc, b)
         np.testing.assert_allclose(got[:, s0:s0 + P], ref[b]["S"], rtol=TOL_SCORE_REL, atol=0)
+
+
+def test_fma_pipe_exp2_against_exact():
+    """The scoring epilogues' polynomial exponential: relative error below
+    2.2e-7 against exact 2^x (fp64) over [-125, 0.5], 2^-125 below that."""
+    x = np.concatenate([np.linspace(-125.0, 0.5, 2_000_001), np.linspace(-1.0, 0.0, 100_001),
+                        [0.0, -0.5, 0.5, -1.0, -124.99, -1000.0, -3e38]]).astype(np.float32)
+    xt = torch.from_numpy(x).cuda()
+    yt = torch.empty_like(xt)
+    tb.tb_diag_exp2(xt, yt)
+    y = yt.cpu().numpy().astype(np.float64)
+    xc = np.maximum(x.astype(np.float64), -125.0)
+    ref = np.exp2(xc)
+    rel = np.abs(y - ref) / ref
+    assert rel.max() < 2.2e-7, (rel.max(), x[np.argmax(rel)])
