@@ -9,21 +9,28 @@
 // (bf16 x bf16 -> fp32 in TMEM). Two passes, because every row needs its
 // global log-sum-exp before any key's score can be summed:
 //
-//  pass 1 (ws_stats_tc)  D[row][key] = Q K^T: each epilogue thread owns one
-//                        window row and folds its keys into a running
-//                        (max, sum of 2^(t - max)) pair;
-//  pass 2 (ws_scores_tc) D[key][row] = K Q^T: each epilogue thread owns one
-//                        key and sums 2^(t - c_row) over the rows, reading
-//                        the key tiles in reverse order so that the tail the
-//                        first pass loaded last is still in L2.
+//  pass 1 (statistics)  D[row][key] = Q K^T: each epilogue thread owns one
+//                       window row (and half of each tile's keys) and folds
+//                       them into a running (max, sum of 2^(t - max)) pair;
+//  pass 2 (votes)       D[key][row] = K Q^T: each epilogue thread owns one key
+//                       (and a quarter of the rows) and sums 2^(t - c_row),
+//                       reading the key tiles in reverse order so that the
+//                       tail pass 1 loaded last is still in L2.
 //
-// Warp roles (640 threads, one CTA per SM): warp 0 issues TMA loads, warp 1
-// issues the MMAs (one elected thread), warp 2 owns the TMEM allocation, and
-// warps 4..19 are the epilogue: four per TMEM lane quadrant, each taking a
-// quarter of the accumulator columns (the epilogue is latency-bound, so it
-// wants many warps). Shared memory holds the
-// window rows once and a 4-stage ring of key tiles; TMEM holds two 256-column
-// accumulators so the MMA of tile t+1 overlaps the epilogue of tile t.
+// One kernel template runs pass 1, pass 2, or both. Both (the default) is a
+// cooperative launch of one CTA per SM: after pass 1 every CTA publishes its
+// per-row partials, meets the others at a grid barrier (bounded wait), and
+// merges the partials of its own KV head into c_row itself; meanwhile its TMA
+// and MMA warps have already moved on to pass 2's first tiles. The fallback,
+// when the grid cannot be co-resident, is pass 1, a merge kernel, then pass 2.
+//
+// Warp roles (576 threads, one CTA per SM): warps 0..15 are the epilogue, four
+// per TMEM lane quadrant, each taking a quarter of the accumulator columns
+// (the epilogue is latency-bound, so it wants many warps); warp 16 issues TMA
+// loads and owns the TMEM allocation; warp 17 issues the MMAs (one thread).
+// Shared memory holds the window rows once and a 4-stage ring of key tiles;
+// TMEM holds two 256-column accumulators so the MMA of tile t+1 overlaps the
+// epilogue of tile t.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -39,16 +46,20 @@ namespace {
 
 constexpr int kTileKeys = 128;
 constexpr int kStages = 4;
-constexpr int kThreads = 640;
-constexpr int kEpiWarp0 = 4;
-constexpr int kEpiWarps = 16;  // four per TMEM lane quadrant, each on a quarter of the columns
+constexpr int kThreads = 576;
+constexpr int kEpiWarps = 16;      // four per TMEM lane quadrant
+constexpr int kProducerWarp = 16;  // TMA issue; also owns the TMEM allocation
+constexpr int kMmaWarp = 17;       // tcgen05.mma issue
 constexpr uint32_t kTmemCols = 512;
 constexpr int kBoxBytes = 128 * 128;  // one TMA box: 128 rows x 64 bf16
 // Of every 32 exponentials an epilogue thread takes, the first kMufuElems go
 // to the MUFU unit and the rest to the FMA pipes (tc::exp2_poly2). Measured on
-// GB300: sending 12 of 32 to the FMA pipes slowed both passes (the epilogue is
-// bound by latency, not by MUFU throughput), so all of them use MUFU.
+// GB300: sending 4 or 8 of 32 to the FMA pipes slowed both passes (they are
+// bound by streaming K, and the epilogue by latency, not by MUFU throughput),
+// so all of them use MUFU.
 constexpr int kMufuElems = 32;
+
+enum : int { kPassStats = 1, kPassVotes = 2, kPassBoth = 3 };
 
 template <int D>
 struct Geo {
@@ -59,8 +70,8 @@ struct Geo {
   static constexpr int kKSteps = D / 16;
   static constexpr int kRingOff = kQBytes;
   static constexpr int kBarOff = kRingOff + kStages * kTileBytes;
-  static constexpr int kCrOff = kBarOff + 1024;
-  static constexpr int kXOff = kCrOff + 256 * 4;       // pass 2: 2 x 3 x 128 partial sums
+  static constexpr int kCrOff = kBarOff + 1024;          // -c_row for 256 rows
+  static constexpr int kXOff = kCrOff + 256 * 4;         // pass 2: 2 x 3 x 128 partial sums
   static constexpr int kMOff = kXOff + 2 * 3 * 128 * 4;  // pass 1: 256 (max, sum) pairs
   static constexpr int kSmem = kMOff + 256 * 8 + 1024;   // + alignment slack
 };
@@ -71,8 +82,12 @@ struct Bars {
   uint64_t tfull[2];
   uint64_t tempty[2];
   uint64_t qfull;
-  uint64_t xfull[2];   // pass 2: the second warpgroup's half sums are in xbuf
-  uint64_t xempty[2];  // pass 2: the first warpgroup consumed them
+  uint64_t xfull[2];  // pass 2: the other quarters' sums are in xbuf
+  uint64_t xempty[2];
+  uint64_t mrg;       // pass 1: the second column halves wrote their (max, sum)
+  uint64_t pub;       // both passes: the CTA's partials are written
+  uint64_t gready;    // both passes: every CTA of the grid published
+  uint64_t crdone;    // -c_row is in shared memory
   uint32_t tmem_base;
   int abort;
 };
@@ -87,11 +102,17 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 struct ItemInfo {
-  int b, g, j0, j1;
+  int b, g, j0, j1_all, j1_pre;
 };
 
-__device__ __forceinline__ ItemInfo locate(const EvictParams& p, int item, bool prefix_only) {
+__device__ __forceinline__ ItemInfo locate(const EvictParams& p, int item) {
   int b = 0;
   while (b + 1 < p.batch && p.req[b + 1].item0 <= item) ++b;
   const EvictReq& rq = p.req[b];
@@ -101,13 +122,52 @@ __device__ __forceinline__ ItemInfo locate(const EvictParams& p, int item, bool 
   it.b = b;
   it.g = local / nch;
   it.j0 = (local % nch) * p.chunk;
-  it.j1 = min(prefix_only ? rq.p : rq.n, it.j0 + p.chunk);
+  it.j1_all = min(rq.n, it.j0 + p.chunk);  // pass 1: every key of the chunk
+  it.j1_pre = min(rq.p, it.j0 + p.chunk);  // pass 2: prefix keys only
   return it;
 }
 
-// Common set-up: barriers and the TMEM allocation. Returns the TMEM base.
-__device__ __forceinline__ uint32_t setup(Bars* bars) {
-  const int warp = threadIdx.x / 32;
+// Byte offset of k-step kk (16 bf16 = 32 B) inside a 128B-swizzled K-major
+// operand made of 64-column boxes.
+__device__ __forceinline__ uint32_t kstep_off(int kk) {
+  return (uint32_t)((kk >> 2) * kBoxBytes + (kk & 3) * 32);
+}
+
+template <int D, int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+    ws_tc(const __grid_constant__ EvictParams p, const __grid_constant__ CUtensorMap tq,
+          const __grid_constant__ CUtensorMap tk, float2* __restrict__ partial,
+          const float* __restrict__ rowc, float* __restrict__ scores, int32_t* __restrict__ status,
+          uint32_t* __restrict__ gsync) {
+  using G = Geo<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* q_s = smem;
+  uint8_t* ring = smem + G::kRingOff;
+  Bars* bars = reinterpret_cast<Bars*>(smem + G::kBarOff);
+  float* ncr = reinterpret_cast<float*>(smem + G::kCrOff);
+  float* xbuf = reinterpret_cast<float*>(smem + G::kXOff);
+  float2* mrg = reinterpret_cast<float2*>(smem + G::kMOff);
+
+  const int item = blockIdx.x;
+  const ItemInfo info = locate(p, item);
+  const EvictReq& rq = p.req[info.b];
+  const int n1 = (MODE & kPassStats) ? (info.j1_all - info.j0 + kTileKeys - 1) / kTileKeys : 0;
+  const int n2 = ((MODE & kPassVotes) && info.j1_pre > info.j0)
+                     ? (info.j1_pre - info.j0 + kTileKeys - 1) / kTileKeys
+                     : 0;
+  if (n1 + n2 == 0) return;  // votes only, and this chunk holds window keys only
+  const int M = p.m_rows;
+  const int RB = M > 128 ? 2 : 1;  // 128-row blocks of the window rows
+  const int NP = (M + 15) & ~15;   // pass 2 MMA N: window rows rounded up to 16
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const size_t segrow = ((size_t)info.b * p.hkv + info.g) * M;
+
+  if (MODE == kPassVotes)
+    for (int r = threadIdx.x; r < 256; r += blockDim.x)
+      ncr[r] = r < M ? -rowc[segrow + r] : -INFINITY;
+
+  // ---- set-up: barriers and the TMEM allocation
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       tc::mbar_init(&bars->full[s], 1);
@@ -116,81 +176,28 @@ __device__ __forceinline__ uint32_t setup(Bars* bars) {
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(&bars->tfull[a], 1);
       tc::mbar_init(&bars->tempty[a], kEpiWarps);
+      tc::mbar_init(&bars->xfull[a], kEpiWarps * 3 / 4);
+      tc::mbar_init(&bars->xempty[a], kEpiWarps / 4);
     }
     tc::mbar_init(&bars->qfull, 1);
-    for (int x = 0; x < 2; ++x) {
-      tc::mbar_init(&bars->xfull[x], kEpiWarps * 3 / 4);
-      tc::mbar_init(&bars->xempty[x], kEpiWarps / 4);
-    }
+    tc::mbar_init(&bars->mrg, kEpiWarps / 2);
+    tc::mbar_init(&bars->pub, kEpiWarps);
+    tc::mbar_init(&bars->gready, 1);
+    tc::mbar_init(&bars->crdone, kEpiWarps);
     bars->abort = 0;
     tc::fence_barrier_init();
   }
-  if (warp == 2) tc::tmem_alloc(&bars->tmem_base, kTmemCols);
+  if (warp == kProducerWarp) tc::tmem_alloc(&bars->tmem_base, kTmemCols);
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
-  return bars->tmem_base;
-}
-
-// Producer and MMA drains + TMEM release, run by every thread at the end.
-__device__ __forceinline__ void teardown(Bars* bars, uint32_t tmem, int issued, int committed,
-                                         int32_t* status) {
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  volatile int* abort = &bars->abort;
-  if (warp == 0 && lane == 0 && *abort) {
-    // wait for the copies still in flight so no copy lands after exit
-    int dummy = 0;
-    tc::mbar_wait(&bars->qfull, 0, &dummy, status);
-    for (int s = 0; s < kStages && s < issued; ++s) {
-      const int last = issued - 1 - ((issued - 1 - s) % kStages);
-      int dummy = 0;
-      tc::mbar_wait(&bars->full[s], (uint32_t)((last / kStages) & 1), &dummy, status);
-    }
-  }
-  if (warp == 1 && lane == 0 && committed > 0) {
-    // the last accumulator commit covers every MMA this thread issued
-    const int last = committed - 1;
-    int dummy = 0;
-    tc::mbar_wait(&bars->tfull[last & 1], (uint32_t)((last >> 1) & 1), &dummy, status);
-  }
-  tc::tc_fence_before();
-  __syncthreads();
-  if (warp == 2) {
-    tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, kTmemCols);
-  }
-}
-
-// ---------------------------------------------------------------------------
-// pass 1: per-row (max, sum) over one chunk of keys
-// ---------------------------------------------------------------------------
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    ws_stats_tc(const __grid_constant__ EvictParams p, const __grid_constant__ CUtensorMap tq,
-                const __grid_constant__ CUtensorMap tk, float2* __restrict__ partial,
-                int32_t* __restrict__ status) {
-  using G = Geo<D>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = align1024(smem_raw);
-  uint8_t* q_s = smem;
-  uint8_t* ring = smem + G::kRingOff;
-  Bars* bars = reinterpret_cast<Bars*>(smem + G::kBarOff);
-  float2* mrg = reinterpret_cast<float2*>(smem + G::kMOff);
-  bool my_ok = false;
-  float my_m = -INFINITY, my_l = 0.f;
-
-  const int item = blockIdx.x;
-  const ItemInfo info = locate(p, item, false);
-  const EvictReq& rq = p.req[info.b];
-  const int ntiles = (info.j1 - info.j0 + kTileKeys - 1) / kTileKeys;
-  const int M = p.m_rows;
-  const int RB = M > 128 ? 2 : 1;
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const uint32_t tmem = setup(bars);
+  const uint32_t tmem = bars->tmem_base;
   volatile int* abort = &bars->abort;
   int issued = 0, committed = 0;
+  const int ntot = n1 + n2;
 
-  if (warp == 0) {
+  if (warp == kProducerWarp) {
+    // ---------------------------------------------------------------- TMA
     if (lane == 0) {
       tc::tma_prefetch_desc(&tq);
       tc::tma_prefetch_desc(&tk);
@@ -201,34 +208,49 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::tma_load_2d(q_s + h * G::kQHalf + rb * kBoxBytes, &tq, h * 64, qrow + rb * 128,
                           &bars->qfull);
       const int krow = (int)((int64_t)info.g * p.kv_rows + rq.kv_off) + info.j0;
-      for (int it = 0; it < ntiles; ++it) {
+      for (int it = 0; it < ntot; ++it) {
         const int s = it % kStages;
+        // pass 1 forward, pass 2 backward
+        const int t = it < n1 ? it : n2 - 1 - (it - n1);
         if (!tc::mbar_wait(&bars->empty[s], ((it / kStages) & 1) ^ 1, abort, status)) break;
         tc::mbar_arrive_expect_tx(&bars->full[s], (uint32_t)G::kTileBytes);
         for (int h = 0; h < G::KH; ++h)
           tc::tma_load_2d(ring + s * G::kTileBytes + h * kBoxBytes, &tk, h * 64,
-                          krow + it * kTileKeys, &bars->full[s]);
+                          krow + t * kTileKeys, &bars->full[s]);
         issued = it + 1;
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------------- MMA
     if (lane == 0 && tc::mbar_wait(&bars->qfull, 0, abort, status)) {
-      constexpr uint32_t idesc = tc::idesc_bf16(128, kTileKeys);
-      for (int it = 0; it < ntiles; ++it) {
+      constexpr uint32_t idesc1 = tc::idesc_bf16(128, kTileKeys);
+      const uint32_t idesc2 = tc::idesc_bf16(128, NP);
+      const uint32_t qbase = tc::smem_addr(q_s);
+      for (int it = 0; it < ntot; ++it) {
         const int s = it % kStages, a = it & 1;
         if (!tc::mbar_wait(&bars->full[s], (it / kStages) & 1, abort, status)) break;
         if (!tc::mbar_wait(&bars->tempty[a], ((it >> 1) & 1) ^ 1, abort, status)) break;
         tc::tc_fence_after();
         const uint32_t kbase = tc::smem_addr(ring + s * G::kTileBytes);
-        const uint32_t qbase = tc::smem_addr(q_s);
+        if (it < n1) {
+          // D[row][key] = Q K^T, one MMA per 128-row block
 #pragma unroll
-        for (int kk = 0; kk < G::kKSteps; ++kk) {
-          const uint32_t off = (uint32_t)((kk >> 2) * kBoxBytes + (kk & 3) * 32);
-          const uint64_t bdesc = tc::sw128_desc(kbase + off);
-          for (int rb = 0; rb < RB; ++rb) {
-            const uint64_t adesc =
-                tc::sw128_desc(qbase + (uint32_t)((kk >> 2) * G::kQHalf + rb * kBoxBytes + (kk & 3) * 32));
-            tc::mma_bf16(tmem + (uint32_t)(a * 256 + rb * 128), adesc, bdesc, idesc, kk > 0);
+          for (int kk = 0; kk < G::kKSteps; ++kk) {
+            const uint64_t bdesc = tc::sw128_desc(kbase + kstep_off(kk));
+            for (int rb = 0; rb < RB; ++rb) {
+              const uint64_t adesc = tc::sw128_desc(
+                  qbase + (uint32_t)((kk >> 2) * G::kQHalf + rb * kBoxBytes + (kk & 3) * 32));
+              tc::mma_bf16(tmem + (uint32_t)(a * 256 + rb * 128), adesc, bdesc, idesc1, kk > 0);
+            }
+          }
+        } else {
+          // D[key][row] = K Q^T over the NP window rows
+#pragma unroll
+          for (int kk = 0; kk < G::kKSteps; ++kk) {
+            const uint64_t adesc = tc::sw128_desc(kbase + kstep_off(kk));
+            const uint64_t bdesc =
+                tc::sw128_desc(qbase + (uint32_t)((kk >> 2) * G::kQHalf + (kk & 3) * 32));
+            tc::mma_bf16(tmem + (uint32_t)(a * 256), adesc, bdesc, idesc2, kk > 0);
           }
         }
         tc::mma_commit(&bars->empty[s]);
@@ -236,48 +258,63 @@ __global__ void __launch_bounds__(kThreads, 1)
         committed = it + 1;
       }
     }
-  } else if (warp >= kEpiWarp0) {
-    // rows: row block wg, TMEM lane quadrant quad; columns: half `half` of the tile
-    const int e = warp - kEpiWarp0, sub = e >> 2, quad = warp & 3;
-    const int wg = sub >> 1, half = sub & 1;
-    const int row = wg * 128 + quad * 32 + lane;
-    const int w = row % p.window;
-    const int vis_end = min(rq.n, rq.p + w + 1);  // keys [0, vis_end) visible to the row
+  } else if (warp < kEpiWarps) {
+    // ---------------------------------------------------------------- epilogue
+    const int sub = warp >> 2, quad = warp & 3;
     const float c = p.scale_log2;
-    float m_run = -INFINITY;
-    float l_run = 0.f, l_comp = 0.f;  // compensated running sum of 2^(t - m_run)
     bool ok = true;
-    for (int it = 0; it < ntiles; ++it) {
-      const int a = it & 1;
-      if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) {
-        ok = false;
-        break;
-      }
-      tc::tc_fence_after();
-      if (wg < RB) {
-        const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(a * 256 + wg * 128);
-        const int key0 = info.j0 + it * kTileKeys;
-        const bool all_vis = key0 + kTileKeys <= rq.p;
-#pragma unroll 1
-        for (int ch = 2 * half; ch < 2 * half + 2; ++ch) {
-          float v[32];
+
+    if (MODE & kPassStats) {
+      // rows: row block wg, TMEM lane quadrant quad; keys: half `half` of each tile
+      const int wg = sub >> 1, half = sub & 1;
+      const int row = wg * 128 + quad * 32 + lane;
+      const int w = row % p.window;
+      const int vis_end = min(rq.n, rq.p + w + 1);  // keys [0, vis_end) visible to the row
+      float m_run = -INFINITY;
+      float l_run = 0.f, l_comp = 0.f;  // compensated running sum of 2^(t - m_run)
+      for (int it = 0; it < n1; ++it) {
+        const int a = it & 1;
+        if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) {
+          ok = false;
+          break;
+        }
+        tc::tc_fence_after();
+        bool released = false;
+        if (wg < RB) {
+          const uint32_t taddr =
+              tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(a * 256 + wg * 128 + half * 64);
+          const int key0 = info.j0 + it * kTileKeys + half * 64;
+          const bool all_vis = info.j0 + (it + 1) * kTileKeys <= rq.p;
+          // this warp's 64 columns of the tile: two TMEM loads, one wait
+          float v[64];
           __syncwarp();
-          tc::tmem_ld32(taddr + ch * 32, v);
+          tc::tmem_ld32(taddr, *reinterpret_cast<float(*)[32]>(v));
+          tc::tmem_ld32(taddr + 32, *reinterpret_cast<float(*)[32]>(v + 32));
           tc::tmem_ld_wait();
+          // the values are in registers: hand the accumulator back to the MMA
+          // warp before computing, so the next-but-one tile's MMAs can start
+          tc::tc_fence_before();
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
+          released = true;
           if (!all_vis) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (key0 + ch * 32 + i >= vis_end) v[i] = -INFINITY;
+            for (int i = 0; i < 64; ++i)
+              if (key0 + i >= vis_end) v[i] = -INFINITY;
           }
-          // chunk max with three-input max (tree of 16 + 5 + 2 + 1 ops)
-          float mt[11];
+          // slab max with three-input max
+          float mt[22];
 #pragma unroll
-          for (int i = 0; i < 10; ++i) mt[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
-          mt[10] = fmaxf(v[30], v[31]);
-          const float mx = tc::max3(tc::max3(mt[0], mt[1], mt[2]), tc::max3(mt[3], mt[4], mt[5]),
-                                    tc::max3(tc::max3(mt[6], mt[7], mt[8]), mt[9], mt[10]));
+          for (int i = 0; i < 21; ++i) mt[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+          mt[21] = v[63];
+          float mu[8];
+#pragma unroll
+          for (int i = 0; i < 7; ++i) mu[i] = tc::max3(mt[3 * i], mt[3 * i + 1], mt[3 * i + 2]);
+          mu[7] = mt[21];
+          const float mx = tc::max3(tc::max3(mu[0], mu[1], mu[2]), tc::max3(mu[3], mu[4], mu[5]),
+                                    fmaxf(mu[6], mu[7]));
           const float m_new = fmaxf(m_run, mx * c);
-          if (m_new != -INFINITY) {  // some key of this chunk is visible
+          if (m_new != -INFINITY) {  // some key of this slab is visible
             if (m_new > m_run) {
               const float sc = fast_exp2(m_run - m_new);
               l_run *= sc;
@@ -288,19 +325,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t cc = tc::pk2(c, c), mm = tc::pk2(-m_run, -m_run);
             uint64_t acc0 = 0, acc1 = 0;
 #pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-              const float2 a = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), cc, mm));
-              const float2 bq = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), cc, mm));
-              float2 ea, eb;
-              if (i < kMufuElems) {
-                ea = make_float2(fast_exp2(a.x), fast_exp2(a.y));
-                eb = make_float2(fast_exp2(bq.x), fast_exp2(bq.y));
+            for (int i = 0; i < 64; i += 4) {
+              const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), cc, mm));
+              const float2 y = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), cc, mm));
+              float2 ex, ey;
+              if ((i & 31) < kMufuElems) {
+                ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+                ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
               } else {
-                ea = tc::exp2_poly2(a.x, a.y);
-                eb = tc::exp2_poly2(bq.x, bq.y);
+                ex = tc::exp2_poly2(x.x, x.y);
+                ey = tc::exp2_poly2(y.x, y.y);
               }
-              acc0 = tc::add2(acc0, tc::pk2(ea.x, ea.y));
-              acc1 = tc::add2(acc1, tc::pk2(eb.x, eb.y));
+              acc0 = tc::add2(acc0, tc::pk2(ex.x, ex.y));
+              acc1 = tc::add2(acc1, tc::pk2(ey.x, ey.y));
             }
             const float2 s01 = tc::upk2(tc::add2(acc0, acc1));
             const float term = (s01.x + s01.y) - l_comp;
@@ -309,178 +346,178 @@ __global__ void __launch_bounds__(kThreads, 1)
             l_run = tsum;
           }
         }
-      }
-      tc::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
-    }
-    // the second column half hands its (max, sum) to the first
-    if (half == 1) mrg[row] = make_float2(ok ? m_run : NAN, l_run);
-    my_ok = ok;
-    my_m = m_run;
-    my_l = l_run;
-  }
-  __syncthreads();
-  if (warp >= kEpiWarp0) {
-    const int e = warp - kEpiWarp0, sub = e >> 2, quad = warp & 3;
-    const int wg = sub >> 1, half = sub & 1;
-    const int row = wg * 128 + quad * 32 + lane;
-    if (half == 0 && wg < RB && row < M) {
-      const float2 o = mrg[row];
-      if (my_ok && !isnan(o.x)) {
-        const float m = fmaxf(my_m, o.x);
-        const float l = (m == -INFINITY) ? 0.f
-                                        : my_l * fast_exp2(my_m - m) + o.y * fast_exp2(o.x - m);
-        partial[(size_t)item * M + row] = make_float2(m, l);
-      }
-    }
-  }
-  teardown(bars, tmem, issued, committed, status);
-}
-
-// ---------------------------------------------------------------------------
-// pass 2: per-key normalised window sum
-// ---------------------------------------------------------------------------
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    ws_scores_tc(const __grid_constant__ EvictParams p, const __grid_constant__ CUtensorMap tq,
-                 const __grid_constant__ CUtensorMap tk, const float* __restrict__ rowc,
-                 float* __restrict__ scores, int32_t* __restrict__ status) {
-  using G = Geo<D>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = align1024(smem_raw);
-  uint8_t* q_s = smem;
-  uint8_t* ring = smem + G::kRingOff;
-  Bars* bars = reinterpret_cast<Bars*>(smem + G::kBarOff);
-  float* cr = reinterpret_cast<float*>(smem + G::kCrOff);
-  float* xbuf = reinterpret_cast<float*>(smem + G::kXOff);
-
-  const int item = blockIdx.x;
-  const ItemInfo info = locate(p, item, true);
-  if (info.j1 <= info.j0) return;  // this chunk holds window keys only
-  const EvictReq& rq = p.req[info.b];
-  const int ntiles = (info.j1 - info.j0 + kTileKeys - 1) / kTileKeys;
-  const int M = p.m_rows;
-  const int NP = (M + 15) & ~15;  // MMA N: window rows rounded up to 16
-  const int RBQ = NP > 128 ? 2 : 1;
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-
-  const float* rc = rowc + ((size_t)info.b * p.hkv + info.g) * M;
-  float* ncr = cr;  // -c_row; -inf for padding rows so that their terms vanish
-  for (int r = threadIdx.x; r < 256; r += blockDim.x) ncr[r] = r < M ? -rc[r] : -INFINITY;
-  const uint32_t tmem = setup(bars);
-  volatile int* abort = &bars->abort;
-  int issued = 0, committed = 0;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      tc::tma_prefetch_desc(&tq);
-      tc::tma_prefetch_desc(&tk);
-      const int qrow = (info.b * p.hq + info.g * p.group) * p.window;
-      tc::mbar_arrive_expect_tx(&bars->qfull, (uint32_t)(RBQ * G::KH * kBoxBytes));
-      for (int h = 0; h < G::KH; ++h)
-        for (int rb = 0; rb < RBQ; ++rb)
-          tc::tma_load_2d(q_s + h * G::kQHalf + rb * kBoxBytes, &tq, h * 64, qrow + rb * 128,
-                          &bars->qfull);
-      const int krow = (int)((int64_t)info.g * p.kv_rows + rq.kv_off) + info.j0;
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % kStages;
-        const int t = ntiles - 1 - it;  // reverse order: the first pass's tail is in L2
-        if (!tc::mbar_wait(&bars->empty[s], ((it / kStages) & 1) ^ 1, abort, status)) break;
-        tc::mbar_arrive_expect_tx(&bars->full[s], (uint32_t)G::kTileBytes);
-        for (int h = 0; h < G::KH; ++h)
-          tc::tma_load_2d(ring + s * G::kTileBytes + h * kBoxBytes, &tk, h * 64,
-                          krow + t * kTileKeys, &bars->full[s]);
-        issued = it + 1;
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0 && tc::mbar_wait(&bars->qfull, 0, abort, status)) {
-      const uint32_t idesc = tc::idesc_bf16(128, NP);
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % kStages, a = it & 1;
-        if (!tc::mbar_wait(&bars->full[s], (it / kStages) & 1, abort, status)) break;
-        if (!tc::mbar_wait(&bars->tempty[a], ((it >> 1) & 1) ^ 1, abort, status)) break;
-        tc::tc_fence_after();
-        const uint32_t kbase = tc::smem_addr(ring + s * G::kTileBytes);
-        const uint32_t qbase = tc::smem_addr(q_s);
-#pragma unroll
-        for (int kk = 0; kk < G::kKSteps; ++kk) {
-          const uint64_t adesc = tc::sw128_desc(kbase + (uint32_t)((kk >> 2) * kBoxBytes + (kk & 3) * 32));
-          const uint64_t bdesc = tc::sw128_desc(qbase + (uint32_t)((kk >> 2) * G::kQHalf + (kk & 3) * 32));
-          tc::mma_bf16(tmem + (uint32_t)(a * 256), adesc, bdesc, idesc, kk > 0);
+        if (!released) {
+          tc::tc_fence_before();
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
         }
-        tc::mma_commit(&bars->empty[s]);
-        tc::mma_commit(&bars->tfull[a]);
-        committed = it + 1;
       }
-    }
-  } else if (warp >= kEpiWarp0) {
-    // keys: TMEM lane quadrant quad; window rows (columns): quarter `sub`
-    const int e = warp - kEpiWarp0, sub = e >> 2, quad = warp & 3;
-    const int key = quad * 32 + lane;  // TMEM lane = key within the tile
-    const float c = p.scale_log2;
-    float* out = scores + (size_t)info.g * p.score_rows + rq.score_off;
-    for (int it = 0; it < ntiles; ++it) {
-      const int a = it & 1;
-      const int t = ntiles - 1 - it;
-      if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) break;
-      tc::tc_fence_after();
-      const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(a * 256);
-      float acc = 0.f;
-#pragma unroll 1
-      for (int ch = 0; ch < 2; ++ch) {
-        const int c0 = sub * 64 + ch * 32;
-        if (c0 >= NP) break;
-        float v[32];
+      // the second column half hands its (max, sum) to the first
+      if (half == 1) {
+        if (ok) mrg[row] = make_float2(m_run, l_run);
         __syncwarp();
-        tc::tmem_ld32(taddr + c0, v);
-        tc::tmem_ld_wait();
-        // 2^(v c - c_row) in packed pairs; -c_row pairs come from shared memory
-        const uint64_t c2 = tc::pk2(c, c);
-        uint64_t a0 = 0, a1 = 0;
-#pragma unroll
-        for (int i = 0; i < 32; i += 4) {
-          const float4 nc = *reinterpret_cast<const float4*>(ncr + c0 + i);
-          const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), c2, tc::pk2(nc.x, nc.y)));
-          const float2 y = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), c2, tc::pk2(nc.z, nc.w)));
-          float2 ex, ey;
-          if (i < kMufuElems) {
-            ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
-            ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
-          } else {
-            ex = tc::exp2_poly2(x.x, x.y);
-            ey = tc::exp2_poly2(y.x, y.y);
-          }
-          a0 = tc::add2(a0, tc::pk2(ex.x, ex.y));
-          a1 = tc::add2(a1, tc::pk2(ey.x, ey.y));
-        }
-        const float2 s01 = tc::upk2(tc::add2(a0, a1));
-        acc += s01.x + s01.y;
-      }
-      tc::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
-      // combine the four quarters of the window rows through a double-buffered
-      // hand-off (bounded mbarrier waits, no named barrier); fixed sum order
-      const int x = it & 1;
-      const uint32_t xph = (uint32_t)((it >> 1) & 1);
-      if (sub > 0) {
-        if (!tc::mbar_wait(&bars->xempty[x], xph ^ 1, abort, status)) break;
-        xbuf[(x * 3 + sub - 1) * 128 + key] = acc;
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&bars->xfull[x]);
+        if (lane == 0) tc::mbar_arrive(&bars->mrg);
       } else {
-        if (!tc::mbar_wait(&bars->xfull[x], xph, abort, status)) break;
-        const int j = info.j0 + t * kTileKeys + key;
-        const float* xb = xbuf + x * 3 * 128;
-        if (j < info.j1) out[j] = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&bars->xempty[x]);
+        ok = ok && tc::mbar_wait(&bars->mrg, 0, abort, status);
+        if (ok && wg < RB && row < M) {
+          const float2 o = mrg[row];
+          const float m = fmaxf(m_run, o.x);
+          const float l =
+              (m == -INFINITY) ? 0.f : l_run * fast_exp2(m_run - m) + o.y * fast_exp2(o.x - m);
+          partial[(size_t)item * M + row] = make_float2(m, l);
+        }
+      }
+    }
+
+    if (MODE == kPassBoth) {
+      // publish this CTA's partials, then meet the grid (one thread waits)
+      __threadfence();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->pub);
+      if (warp == 0 && lane == 0) {
+        if (tc::mbar_wait(&bars->pub, 0, abort, status) && !*abort) {
+          __threadfence();
+          atomicAdd(gsync, 1u);
+          const uint64_t t0 = tc::globaltimer();
+          while (ld_acquire(gsync) < gridDim.x) {
+            if (*abort) break;
+            if (tc::globaltimer() - t0 > tc::kWaitNs) {
+              *abort = 1;
+              atomicOr(status, kStatusTimeout);
+              break;
+            }
+            __nanosleep(64);
+          }
+        }
+        tc::mbar_arrive(&bars->gready);  // also on abort: the waiters then see the flag
+      }
+      ok = ok && tc::mbar_wait(&bars->gready, 0, abort, status) && !*abort;
+      // merge every chunk of this (request, KV head) into -c_row
+      if (ok) {
+        const int nch = (rq.n + p.chunk - 1) / p.chunk;
+        const size_t it0 = (size_t)rq.item0 + (size_t)info.g * nch;
+        for (int r = threadIdx.x; r < 256; r += kEpiWarps * 32) {
+          float v = -INFINITY;
+          if (r < M) {
+            float m = -INFINITY;
+            for (int ch = 0; ch < nch; ++ch) m = fmaxf(m, __ldcg(&partial[(it0 + ch) * M + r]).x);
+            float l = 0.f, comp = 0.f;  // compensated sum
+            for (int ch = 0; ch < nch; ++ch) {
+              const float2 pv = __ldcg(&partial[(it0 + ch) * M + r]);
+              if (pv.y > 0.f) {
+                const float term = pv.y * exp2f(pv.x - m) - comp;
+                const float t = l + term;
+                comp = (t - l) - term;
+                l = t;
+              }
+            }
+            v = -(m + log2f(l));
+          }
+          ncr[r] = v;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->crdone);
+      ok = ok && tc::mbar_wait(&bars->crdone, 0, abort, status);
+    }
+
+    if ((MODE & kPassVotes) && ok) {
+      // keys: TMEM lane quadrant quad; window rows (columns): quarter `sub`
+      const int key = quad * 32 + lane;  // TMEM lane = key within the tile
+      float* out = scores + (size_t)info.g * p.score_rows + rq.score_off;
+      for (int it2 = 0; it2 < n2; ++it2) {
+        const int it = n1 + it2;
+        const int a = it & 1;
+        const int t = n2 - 1 - it2;
+        if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) break;
+        tc::tc_fence_after();
+        const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(a * 256);
+        float acc = 0.f;
+        bool released = false;
+        const int c0 = sub * 64;
+        if (c0 < NP) {
+          // this warp's (up to) 64 window-row columns: two TMEM loads, one wait
+          float v[64];
+          __syncwarp();
+          tc::tmem_ld32(taddr + c0, *reinterpret_cast<float(*)[32]>(v));
+          if (c0 + 32 < NP) tc::tmem_ld32(taddr + c0 + 32, *reinterpret_cast<float(*)[32]>(v + 32));
+          tc::tmem_ld_wait();
+          tc::tc_fence_before();
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
+          released = true;
+          const int nv = c0 + 32 < NP ? 64 : 32;
+          // 2^(v c - c_row) in packed pairs; -c_row pairs come from shared memory
+          const uint64_t c2 = tc::pk2(c, c);
+          uint64_t a0 = 0, a1 = 0;
+#pragma unroll
+          for (int i = 0; i < 64; i += 4) {
+            if (i >= nv) break;
+            const float4 nc = *reinterpret_cast<const float4*>(ncr + c0 + i);
+            const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), c2, tc::pk2(nc.x, nc.y)));
+            const float2 y =
+                tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), c2, tc::pk2(nc.z, nc.w)));
+            float2 ex, ey;
+            if ((i & 31) < kMufuElems) {
+              ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+              ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
+            } else {
+              ex = tc::exp2_poly2(x.x, x.y);
+              ey = tc::exp2_poly2(y.x, y.y);
+            }
+            a0 = tc::add2(a0, tc::pk2(ex.x, ex.y));
+            a1 = tc::add2(a1, tc::pk2(ey.x, ey.y));
+          }
+          const float2 s01 = tc::upk2(tc::add2(a0, a1));
+          acc = s01.x + s01.y;
+        }
+        if (!released) {
+          tc::tc_fence_before();
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
+        }
+        // combine the four quarters of the window rows through a double-buffered
+        // hand-off (bounded mbarrier waits, no named barrier); fixed sum order
+        const int x = it2 & 1;
+        const uint32_t xph = (uint32_t)((it2 >> 1) & 1);
+        if (sub > 0) {
+          if (!tc::mbar_wait(&bars->xempty[x], xph ^ 1, abort, status)) break;
+          xbuf[(x * 3 + sub - 1) * 128 + key] = acc;
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&bars->xfull[x]);
+        } else {
+          if (!tc::mbar_wait(&bars->xfull[x], xph, abort, status)) break;
+          const int j = info.j0 + t * kTileKeys + key;
+          const float* xb = xbuf + x * 3 * 128;
+          if (j < info.j1_pre) out[j] = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&bars->xempty[x]);
+        }
       }
     }
   }
-  teardown(bars, tmem, issued, committed, status);
+
+  // ---- teardown: drain what is still in flight, release TMEM
+  if (warp == kProducerWarp && lane == 0 && *abort) {
+    int dummy = 0;
+    tc::mbar_wait(&bars->qfull, 0, &dummy, status);
+    for (int s = 0; s < kStages && s < issued; ++s) {
+      const int last = issued - 1 - ((issued - 1 - s) % kStages);
+      tc::mbar_wait(&bars->full[s], (uint32_t)((last / kStages) & 1), &dummy, status);
+    }
+  }
+  if (warp == kMmaWarp && lane == 0 && committed > 0) {
+    // the last accumulator commit covers every MMA this thread issued
+    const int last = committed - 1;
+    int dummy = 0;
+    tc::mbar_wait(&bars->tfull[last & 1], (uint32_t)((last >> 1) & 1), &dummy, status);
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == kProducerWarp) {
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, kTmemCols);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -500,8 +537,65 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-bool make_map(CUtensorMap* map, const void* base, int d, uint64_t rows) {
-  return make_bf16_map(map, base, d, rows, 128);
+// CTAs of the fused kernel that fit on the current device at once (cached).
+int coresident_ctas(const void* kernel, int smem, int slot) {
+  constexpr int kMaxDev = 64;
+  static int cache[kMaxDev][2] = {};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[dev][slot] == 0) {
+    int sms = 0, per_sm = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, smem) !=
+            cudaSuccess)
+      return 0;
+    cache[dev][slot] = sms * per_sm;
+  }
+  return cache[dev][slot];
+}
+
+template <int D>
+cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const CUtensorMap& tk,
+                            float* scores, float2* partial, float* rowc, int32_t* status,
+                            cudaStream_t s) {
+  using Gm = Geo<D>;
+  uint32_t* gsync = reinterpret_cast<uint32_t*>(status) + kGridSyncWord;
+  auto fused = ws_tc<D, kPassBoth>;
+  cudaError_t e =
+      cudaFuncSetAttribute(fused, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
+  if (e != cudaSuccess) return e;
+  if (pt.items <= coresident_ctas(reinterpret_cast<const void*>(fused), Gm::kSmem, D == 128)) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)pt.items, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = Gm::kSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, fused, pt, tq, tk, partial, (const float*)rowc, scores, status,
+                           gsync);
+    count_launches(1);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+  }
+  // fallback: the passes as separate launches with the merge kernel between
+  auto stats = ws_tc<D, kPassStats>;
+  auto votes = ws_tc<D, kPassVotes>;
+  e = cudaFuncSetAttribute(stats, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(votes, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
+  if (e != cudaSuccess) return e;
+  stats<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync);
+  e = launch_window_combine(pt, partial, rowc, s);
+  if (e != cudaSuccess) return e;
+  votes<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync);
+  count_launches(2);
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -520,27 +614,6 @@ bool make_bf16_map(CUtensorMap* map, const void* base, int d, uint64_t rows, int
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-namespace {
-
-template <int D>
-cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const CUtensorMap& tk,
-                            float* scores, float2* partial, float* rowc, int32_t* status,
-                            cudaStream_t s) {
-  using Gm = Geo<D>;
-  cudaError_t e = cudaFuncSetAttribute(ws_stats_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Gm::kSmem);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(ws_scores_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
-  if (e != cudaSuccess) return e;
-  ws_stats_tc<D><<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, status);
-  launch_window_combine(pt, partial, rowc, s);
-  ws_scores_tc<D><<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, rowc, scores, status);
-  count_launches(2);
-  return cudaGetLastError();
-}
-
-}  // namespace
-
 bool window_scores_tc_supported(const EvictParams& p) {
   const uint64_t krows = (uint64_t)p.hkv * (uint64_t)p.kv_rows;
   const uint64_t qrows = (uint64_t)p.batch * p.hq * p.window;
@@ -553,7 +626,8 @@ bool window_scores_tc_supported(const EvictParams& p) {
 EvictParams tc_item_params(const EvictParams& p) {
   EvictParams pt = p;
   int64_t tiles = 0;
-  for (int b = 0; b < p.batch; ++b) tiles += (int64_t)p.hkv * ((p.req[b].n + kTileKeys - 1) / kTileKeys);
+  for (int b = 0; b < p.batch; ++b)
+    tiles += (int64_t)p.hkv * ((p.req[b].n + kTileKeys - 1) / kTileKeys);
   int64_t per_item = (tiles + 151) / 152;
   if (per_item < 2) per_item = 2;  // >= the SIMT chunk, so the workspace stays large enough
   pt.chunk = (int32_t)(per_item * kTileKeys);
@@ -573,7 +647,7 @@ cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, con
   CUtensorMap tq, tk;
   const uint64_t qrows = (uint64_t)p.batch * p.hq * p.window;
   const uint64_t krows = (uint64_t)p.hkv * p.kv_rows;
-  if (!make_map(&tq, q_win, p.d, qrows) || !make_map(&tk, K, p.d, krows))
+  if (!make_bf16_map(&tq, q_win, p.d, qrows, 128) || !make_bf16_map(&tk, K, p.d, krows, 128))
     return cudaErrorInvalidValue;
   return p.d == 64 ? launch_tc_typed<64>(pt, tq, tk, scores, partial, rowc, status, s)
                    : launch_tc_typed<128>(pt, tq, tk, scores, partial, rowc, status, s);

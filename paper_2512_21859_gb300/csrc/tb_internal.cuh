@@ -15,8 +15,11 @@ enum : int32_t {
   kStatusRange = 2,    // a device-side range check fired
 };
 
-// Bytes reserved at the start of each workspace for the status word.
+// Bytes reserved at the start of each workspace for the status word (word 0)
+// and the grid-barrier counter of the fused scoring kernel (word
+// kGridSyncWord); all of it is zeroed at the start of every call.
 constexpr size_t kStatusBytes = 256;
+constexpr int kGridSyncWord = 16;
 
 // Largest G*W (window rows of one KV-head group) the scoring kernels take.
 constexpr int kMaxWindowRows = 1024;
