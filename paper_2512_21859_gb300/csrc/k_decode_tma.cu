@@ -5,7 +5,7 @@
 // softmax over the request's first len keys, attention definition of
 // "FLOPs-based Modeling"), organised for HBM bandwidth: each CTA takes one
 // (request, KV head, key split) and streams its K and V rows through a
-// 3-stage ring of 64-key tiles that one thread fills with 2-D TMA copies
+// 6-stage ring of 64-key tiles that one thread fills with 2-D TMA copies
 // (128-byte swizzle, so ldmatrix reads are free of bank conflicts). The G
 // query heads of the group share every tile, so each K/V byte is read from
 // HBM once per decode step.
@@ -32,10 +32,11 @@
 namespace tb {
 namespace {
 
-constexpr int kThreads = 128;
-constexpr int kTile = 64;
-constexpr int kStages = 3;
-constexpr int kBox = 64 * 128;  // 64 rows x 128 B
+constexpr int kWarps = 8;
+constexpr int kThreads = kWarps * 32;
+constexpr int kTile = kWarps * 16;  // keys per tile: 16 per warp
+constexpr int kStages = 3;          // one CTA per SM, 3 x 64 KB in flight
+constexpr int kBox = kTile * 128;   // one TMA box: kTile rows x 128 B
 
 template <int D>
 struct DGeo {
@@ -43,8 +44,10 @@ struct DGeo {
   static constexpr int kStageBytes = 2 * KH * kBox;  // K and V halves of one tile
   static constexpr int kRing = kStages * kStageBytes;
   // after the key loop the ring holds the cross-warp merge: O, m, l per warp
-  static constexpr int kMergeO = 4 * 16 * D * 4;
-  static_assert(kMergeO + 4 * 16 * 8 <= kRing, "merge area must fit in the ring");
+  // (rows padded by 8 floats so the fragment stores hit distinct banks)
+  static constexpr int kDS = D + 8;
+  static constexpr int kMergeO = kWarps * 16 * kDS * 4;
+  static_assert(kMergeO + kWarps * 16 * 8 <= kRing, "merge area must fit in the ring");
   static constexpr int kMaxSplits = kRing / (16 * 4);  // weights table [G <= 16][splits]
   static constexpr int kBarOff = kRing;
   static constexpr int kSmem = kBarOff + 64 + 1024;  // + alignment slack
@@ -99,7 +102,7 @@ __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
 }
 
 template <int D, int G>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
     decode_tma(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tk,
                const __grid_constant__ CUtensorMap tv, const uint16_t* __restrict__ q,
                const int32_t* __restrict__ lens, float* __restrict__ part_o,
@@ -201,15 +204,25 @@ __global__ void __launch_bounds__(kThreads, 2)
       // ---- S = Q K^T over this warp's 16 keys
       float sc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
       {
+        // even and odd k-steps accumulate separately: two short dependency
+        // chains per n-tile instead of one long one
+        float so[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
         const int krow = kb + (lane & 7) + ((lane >> 4) << 3);
         const int ksel = (lane >> 3) & 1;
 #pragma unroll
-        for (int kk = 0; kk < KS; ++kk) {
-          uint32_t bk[4];
+        for (int kk = 0; kk < KS; kk += 2) {
+          uint32_t bk[4], bk2[4];
           ldsm_x4(kst + sw_off(krow, 2 * kk + ksel), bk);
+          ldsm_x4(kst + sw_off(krow, 2 * kk + 2 + ksel), bk2);
           mma_16816(sc[0], aq[kk], bk[0], bk[1]);
           mma_16816(sc[1], aq[kk], bk[2], bk[3]);
+          mma_16816(so[0], aq[kk + 1], bk2[0], bk2[1]);
+          mma_16816(so[1], aq[kk + 1], bk2[2], bk2[3]);
         }
+#pragma unroll
+        for (int n = 0; n < 2; ++n)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) sc[n][e] += so[n][e];
       }
       // ---- online softmax per row (r0: elements 0,1; r0 + 8: elements 2,3)
       float corr[2];
@@ -303,15 +316,21 @@ __global__ void __launch_bounds__(kThreads, 2)
     l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 1);
     l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 2);
   }
-  float* mo = reinterpret_cast<float*>(smem);                // [4][16][D]
-  float* mml = reinterpret_cast<float*>(smem + Gm::kMergeO);  // [4][16][2]
+  constexpr int DS = Gm::kDS;
+  float* mo = reinterpret_cast<float*>(smem);                // [kWarps][16][DS]
+  float* mml = reinterpret_cast<float*>(smem + Gm::kMergeO);  // [kWarps][16][2]
+  // only the G real query rows of the 16-row MMA tile are kept
+  if (r0 < G) {
 #pragma unroll
-  for (int n = 0; n < NT; ++n) {
-    const int dim = n * 8 + 2 * qd;
-    mo[(warp * 16 + r0) * D + dim] = o[n][0];
-    mo[(warp * 16 + r0) * D + dim + 1] = o[n][1];
-    mo[(warp * 16 + r0 + 8) * D + dim] = o[n][2];
-    mo[(warp * 16 + r0 + 8) * D + dim + 1] = o[n][3];
+    for (int n = 0; n < NT; ++n)
+      *reinterpret_cast<float2*>(mo + (warp * 16 + r0) * DS + n * 8 + 2 * qd) =
+          make_float2(o[n][0], o[n][1]);
+  }
+  if (r0 + 8 < G) {
+#pragma unroll
+    for (int n = 0; n < NT; ++n)
+      *reinterpret_cast<float2*>(mo + (warp * 16 + r0 + 8) * DS + n * 8 + 2 * qd) =
+          make_float2(o[n][2], o[n][3]);
   }
   if (qd == 0) {
     mml[(warp * 16 + r0) * 2] = m_run[0];
@@ -324,16 +343,16 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int h = e / D, dim = e % D;
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) M = fmaxf(M, mml[(w * 16 + h) * 2]);
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mml[(w * 16 + h) * 2]);
     float L = 0.f, O = 0.f;
     if (M != -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
+      for (int w = 0; w < kWarps; ++w) {
         const float mw = mml[(w * 16 + h) * 2];
         if (mw != -INFINITY) {
           const float wt = fast_exp2(mw - M);
           L = fmaf(mml[(w * 16 + h) * 2 + 1], wt, L);
-          O = fmaf(mo[(w * 16 + h) * D + dim], wt, O);
+          O = fmaf(mo[(w * 16 + h) * DS + dim], wt, O);
         }
       }
     }

@@ -1,9 +1,9 @@
 // Gather / compaction of the retained K and V rows.
 //
 //   Kc[g][out_off_b + r] = K[g][kv_off_b + idx[g][idx_off_b + r]],  r < R_b,
-// and the same for V: pure bit copies in 16-byte vectors. One warp moves one
-// retained row of K and the matching row of V; a row is d * elem bytes
-// (128..512 B), so each 16-byte lane access is part of a fully used sector.
+// and the same for V: pure bit copies in 16-byte vectors. A row is d * elem
+// bytes (128..512 B), so each 16-byte lane access is part of a fully used
+// sector.
 #include <cuda_runtime.h>
 
 #include "tb_internal.cuh"
@@ -12,36 +12,51 @@ namespace tb {
 namespace {
 
 constexpr int kGatherThreads = 256;
-constexpr int kRowsPerWarp = 4;
+constexpr int kRowsPerWarp = 8;
+constexpr int kMaxVecPerLane = 16;  // kRowsPerWarp * 2 rows * up to 32 vectors / 32 lanes
 
+// Each warp moves kRowsPerWarp retained rows of K and the matching rows of V:
+// first every lane issues all of its 16-byte loads, then all of its stores,
+// so that each lane keeps several independent loads in flight.
+template <int VPR>
 __global__ void __launch_bounds__(kGatherThreads) gather_kernel(
     const __grid_constant__ EvictParams p, const int32_t* __restrict__ idx,
     const uint4* __restrict__ K, const uint4* __restrict__ V, uint4* __restrict__ Kc,
-    uint4* __restrict__ Vc, int vec_per_row) {
+    uint4* __restrict__ Vc) {
+  constexpr int kVecs = kRowsPerWarp * 2 * VPR;  // vectors a warp moves
+  constexpr int kPerLane = kVecs / 32;
+  static_assert(kPerLane <= kMaxVecPerLane, "too many vectors per lane");
   const int b = blockIdx.y, g = blockIdx.z;
   const EvictReq& rq = p.req[b];
   const int R = rq.k + p.window;
   const int lane = threadIdx.x & 31;
-  const int warp_global = (blockIdx.x * kGatherThreads + threadIdx.x) >> 5;
+  const int r0 = ((blockIdx.x * kGatherThreads + threadIdx.x) >> 5) * kRowsPerWarp;
+  if (r0 >= R) return;
   const int32_t* ig = idx + (size_t)g * p.idx_rows + rq.idx_off;
-  const size_t src_base = ((size_t)g * p.kv_rows + rq.kv_off) * vec_per_row;
-  const size_t dst_base = ((size_t)g * p.out_rows + rq.out_off) * vec_per_row;
-  for (int rr = 0; rr < kRowsPerWarp; ++rr) {
-    const int r = warp_global * kRowsPerWarp + rr;
-    if (r >= R) return;
-    const int j = __ldg(ig + r);
-    if (j < 0 || j >= rq.n) continue;
-    const uint4* ks = K + src_base + (size_t)j * vec_per_row;
-    const uint4* vs = V + src_base + (size_t)j * vec_per_row;
-    uint4* kd = Kc + dst_base + (size_t)r * vec_per_row;
-    uint4* vd = Vc + dst_base + (size_t)r * vec_per_row;
-    for (int v = lane; v < 2 * vec_per_row; v += 32) {
-      if (v < vec_per_row) {
-        kd[v] = __ldg(ks + v);
-      } else {
-        vd[v - vec_per_row] = __ldg(vs + v - vec_per_row);
-      }
+  const size_t src_base = ((size_t)g * p.kv_rows + rq.kv_off) * VPR;
+  const size_t dst_base = ((size_t)g * p.out_rows + rq.out_off) * VPR;
+  uint4 buf[kPerLane];
+  bool ok[kPerLane];
+#pragma unroll
+  for (int i = 0; i < kPerLane; ++i) {
+    const int v = lane + 32 * i;
+    const int rr = v / (2 * VPR), w = v % (2 * VPR);
+    const int r = r0 + rr;
+    int j = -1;
+    if (r < R) j = __ldg(ig + r);
+    ok[i] = r < R && j >= 0 && j < rq.n;
+    if (ok[i]) {
+      const uint4* src = (w < VPR ? K : V) + src_base + (size_t)j * VPR + (w < VPR ? w : w - VPR);
+      buf[i] = __ldg(src);
     }
+  }
+#pragma unroll
+  for (int i = 0; i < kPerLane; ++i) {
+    if (!ok[i]) continue;
+    const int v = lane + 32 * i;
+    const int rr = v / (2 * VPR), w = v % (2 * VPR);
+    uint4* dst = (w < VPR ? Kc : Vc) + dst_base + (size_t)(r0 + rr) * VPR + (w < VPR ? w : w - VPR);
+    *dst = buf[i];
   }
 }
 
@@ -55,9 +70,16 @@ cudaError_t launch_gather(const EvictParams& p, const int32_t* idx, const void* 
   const int bx = (p.max_r + rows_per_block - 1) / rows_per_block;
   if (bx == 0) return cudaSuccess;
   dim3 grid(bx, p.batch, p.hkv);
-  gather_kernel<<<grid, kGatherThreads, 0, s>>>(
-      p, idx, static_cast<const uint4*>(K), static_cast<const uint4*>(V),
-      static_cast<uint4*>(Kc), static_cast<uint4*>(Vc), vec_per_row);
+  const uint4* k4 = static_cast<const uint4*>(K);
+  const uint4* v4 = static_cast<const uint4*>(V);
+  uint4* kc4 = static_cast<uint4*>(Kc);
+  uint4* vc4 = static_cast<uint4*>(Vc);
+  switch (vec_per_row) {
+    case 8: gather_kernel<8><<<grid, kGatherThreads, 0, s>>>(p, idx, k4, v4, kc4, vc4); break;
+    case 16: gather_kernel<16><<<grid, kGatherThreads, 0, s>>>(p, idx, k4, v4, kc4, vc4); break;
+    case 32: gather_kernel<32><<<grid, kGatherThreads, 0, s>>>(p, idx, k4, v4, kc4, vc4); break;
+    default: return cudaErrorInvalidValue;
+  }
   count_launches(1);
   return cudaGetLastError();
 }

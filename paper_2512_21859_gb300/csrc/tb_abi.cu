@@ -178,14 +178,14 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
     p->cache_cap[b] = (int32_t)d->cache_cap[b];
   }
   // Split the keys so that about one CTA per SM of a 152-SM part runs, in
-  // whole 64-key tiles (each CTA keeps three tiles in flight).
+  // whole 128-key tiles (each CTA keeps three tiles in flight).
   const int64_t target = 152;
   const int64_t units = (int64_t)d->batch * d->hkv;
   int64_t splits = (target + units - 1) / units;
-  const int64_t max_splits = (d->max_len + 63) / 64;
+  const int64_t max_splits = (d->max_len + 127) / 128;
   splits = std::max<int64_t>(1, std::min(splits, max_splits));
   int64_t split_len = (d->max_len + splits - 1) / splits;
-  split_len = (split_len + 63) / 64 * 64;
+  split_len = (split_len + 127) / 128 * 128;
   splits = (d->max_len + split_len - 1) / split_len;
   p->splits = (int32_t)splits;
   p->split_len = (int32_t)split_len;
