@@ -83,15 +83,20 @@ struct Bars {
   uint64_t tfull[2];
   uint64_t tempty[2];
   uint64_t qfull;
-  uint64_t xfull[2];  // pass 2: the other quarters' sums are in xbuf
-  uint64_t xempty[2];
+  uint64_t xfull[2][4];  // pass 2, per lane quadrant: the other quarters' sums are in xbuf
+  uint64_t xempty[2][4];
   uint64_t mrg;       // pass 1: the second column halves wrote their (max, sum)
   uint64_t pub;       // both passes: the CTA's partials are written
   uint64_t gready;    // both passes: every CTA of the grid published
   uint64_t crdone;    // -c_row is in shared memory
   uint32_t tmem_base;
   int abort;
+  int codes[8];   // tile code of the it-th tile the producer claimed, at [it % 8]
+  int accode[2];  // the MMA warp's copy for the accumulator it fills
 };
+
+// Tile codes: t >= 0 is pass 1 tile t, -2 - t is pass 2 tile t, kNoTile ends.
+constexpr int kNoTile = -1;
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -110,7 +115,8 @@ __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
 }
 
 struct ItemInfo {
-  int b, g, j0, j1_all, j1_pre;
+  int b, g;      // request, KV head
+  int ch, nch;   // this CTA's index among the (request, KV head)'s CTAs, their count
 };
 
 __device__ __forceinline__ ItemInfo locate(const EvictParams& p, int item) {
@@ -122,9 +128,8 @@ __device__ __forceinline__ ItemInfo locate(const EvictParams& p, int item) {
   ItemInfo it;
   it.b = b;
   it.g = local / nch;
-  it.j0 = (local % nch) * p.chunk;
-  it.j1_all = min(rq.n, it.j0 + p.chunk);  // pass 1: every key of the chunk
-  it.j1_pre = min(rq.p, it.j0 + p.chunk);  // pass 2: prefix keys only
+  it.ch = local % nch;
+  it.nch = nch;
   return it;
 }
 
@@ -185,12 +190,38 @@ __device__ __forceinline__ void mma_tile_steps(bool stats, int rb_count, uint32_
     mma_stats_steps<D, 1, K0, K1>(d_tmem, qdesc, kdesc, on);
 }
 
+// sum over i < NV of 2^(v[i] c + bias[i]) in packed pairs, two packed
+// accumulators; the biases (-c_row of each window row) come from shared memory
+template <int NV>
+__device__ __forceinline__ float vote_sum(const float (&v)[64], float c, const float* bias) {
+  const uint64_t c2 = tc::pk2(c, c);
+  uint64_t a0 = 0, a1 = 0;
+#pragma unroll
+  for (int i = 0; i < NV; i += 4) {
+    const float4 nc = *reinterpret_cast<const float4*>(bias + i);
+    const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), c2, tc::pk2(nc.x, nc.y)));
+    const float2 y = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), c2, tc::pk2(nc.z, nc.w)));
+    float2 ex, ey;
+    if ((i & 31) < kMufuElems) {
+      ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+      ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
+    } else {
+      ex = tc::exp2_poly2(x.x, x.y);
+      ey = tc::exp2_poly2(y.x, y.y);
+    }
+    a0 = tc::add2(a0, tc::pk2(ex.x, ex.y));
+    a1 = tc::add2(a1, tc::pk2(ey.x, ey.y));
+  }
+  const float2 s01 = tc::upk2(tc::add2(a0, a1));
+  return s01.x + s01.y;
+}
+
 template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     ws_tc(const __grid_constant__ EvictParams p, const __grid_constant__ CUtensorMap tq,
           const __grid_constant__ CUtensorMap tk, float2* __restrict__ partial,
           const float* __restrict__ rowc, float* __restrict__ scores, int32_t* __restrict__ status,
-          uint32_t* __restrict__ gsync) {
+          uint32_t* __restrict__ gsync, int32_t* __restrict__ tilectr) {
   using G = Geo<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
@@ -204,11 +235,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int item = blockIdx.x;
   const ItemInfo info = locate(p, item);
   const EvictReq& rq = p.req[info.b];
-  const int n1 = (MODE & kPassStats) ? (info.j1_all - info.j0 + kTileKeys - 1) / kTileKeys : 0;
-  const int n2 = ((MODE & kPassVotes) && info.j1_pre > info.j0)
-                     ? (info.j1_pre - info.j0 + kTileKeys - 1) / kTileKeys
-                     : 0;
-  if (n1 + n2 == 0) return;  // votes only, and this chunk holds window keys only
+  // Key tiles of this (request, KV head): pass 1 all N keys, pass 2 the P
+  // prefix keys. Its CTAs claim them from two counters in the workspace, so
+  // a CTA that runs slower takes fewer tiles (a static split left the grid
+  // barrier waiting ~10 us for the slowest CTA).
+  const int nt1 = (MODE & kPassStats) ? (rq.n + kTileKeys - 1) / kTileKeys : 0;
+  const int nt2 = (MODE & kPassVotes) ? (rq.p + kTileKeys - 1) / kTileKeys : 0;
+  if (nt1 + nt2 == 0) return;
   const int M = p.m_rows;
   const int RB = M > 128 ? 2 : 1;  // 128-row blocks of the window rows
   const int NP = (M + 15) & ~15;   // pass 2 MMA N: window rows rounded up to 16
@@ -228,8 +261,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(&bars->tfull[a], 1);
       tc::mbar_init(&bars->tempty[a], kEpiWarps);
-      tc::mbar_init(&bars->xfull[a], kEpiWarps * 3 / 4);
-      tc::mbar_init(&bars->xempty[a], kEpiWarps / 4);
+      for (int qd = 0; qd < 4; ++qd) {
+        tc::mbar_init(&bars->xfull[a][qd], 3);
+        tc::mbar_init(&bars->xempty[a][qd], 1);
+      }
     }
     tc::mbar_init(&bars->qfull, 1);
     tc::mbar_init(&bars->mrg, kEpiWarps / 2);
@@ -246,7 +281,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bars->tmem_base;
   volatile int* abort = &bars->abort;
   int issued = 0, committed = 0;
-  const int ntot = n1 + n2;
 
   if (warp == kProducerWarp) {
     // ---------------------------------------------------------------- TMA
@@ -259,17 +293,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int rb = 0; rb < RB; ++rb)
           tc::tma_load_2d(q_s + h * G::kQHalf + rb * kBoxBytes, &tq, h * 64, qrow + rb * 128,
                           &bars->qfull);
-      const int krow = (int)((int64_t)info.g * p.kv_rows + rq.kv_off) + info.j0;
-      for (int it = 0; it < ntot; ++it) {
+      const int krow = (int)((int64_t)info.g * p.kv_rows + rq.kv_off);
+      int* ctr = tilectr + 2 * (info.b * p.hkv + info.g);
+      // pass 1 tiles in rising order, then pass 2 tiles from the top, so that
+      // pass 2 starts on the tiles pass 1 loaded last (still in L2). A CTA's
+      // first tile of each pass is its own index among the CTAs of the
+      // (request, KV head); later claims count on from there, each issued one
+      // tile ahead so that its round trip overlaps a wait.
+      bool second = nt1 == 0;
+      int claim = info.ch;
+      for (int it = 0;; ++it) {
         const int s = it % kStages;
-        // pass 1 forward, pass 2 backward
-        const int t = it < n1 ? it : n2 - 1 - (it - n1);
         if (!tc::mbar_wait(&bars->empty[s], ((it / kStages) & 1) ^ 1, abort, status)) break;
+        if (!second && claim >= nt1) {
+          // a stats-only launch leaves the pass 2 counter to the votes launch
+          second = true;
+          claim = nt2 > 0 ? info.ch : 0;
+        }
+        const int t = second ? (claim < nt2 ? nt2 - 1 - claim : -1) : claim;
+        const int code = t < 0 ? kNoTile : (second ? -2 - t : t);
+        bars->codes[it & 7] = code;
+        if (code == kNoTile) {
+          tc::mbar_arrive(&bars->full[s]);  // no copy: the consumers see the end
+          break;
+        }
         tc::mbar_arrive_expect_tx(&bars->full[s], (uint32_t)G::kTileBytes);
         for (int h = 0; h < G::KH; ++h)
           tc::tma_load_2d(ring + s * G::kTileBytes + h * kBoxBytes, &tk, h * 64,
                           krow + t * kTileKeys, &bars->full[s]);
         issued = it + 1;
+        claim = info.nch + atomicAdd(ctr + (second ? 1 : 0), 1);
       }
     }
   } else if (warp == kMmaWarp) {
@@ -281,19 +334,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t idesc2 = tc::idesc_bf16(128, NP);
       const uint64_t qdesc = tc::sw128_desc(tc::smem_addr(q_s));
       const uint64_t rdesc = tc::sw128_desc(tc::smem_addr(ring));
-      for (int it = 0; it < ntot; ++it) {
+      for (int it = 0;; ++it) {
         const int s = it % kStages, a = it & 1;
         const bool ready = tc::mbar_wait(&bars->full[s], (it / kStages) & 1, abort, status) &&
                            tc::mbar_wait(&bars->tempty[a], ((it >> 1) & 1) ^ 1, abort, status);
         if (!__all_sync(0xffffffffu, ready)) break;
         tc::tc_fence_after();
+        // the tile code travels with the accumulator to the epilogue
+        const int code = reinterpret_cast<volatile int*>(bars->codes)[it & 7];
+        if (lane == 0) reinterpret_cast<volatile int*>(bars->accode)[a] = code;
+        __threadfence_block();
         const uint32_t on = tc::elect_one();
-        const uint64_t kdesc = desc_plus(rdesc, (uint32_t)(s * G::kTileBytes));
-        const uint32_t dt = tmem + (uint32_t)(a * 256);
-        mma_tile_steps<D, 0, G::kKSteps>(it < n1, RB, dt, qdesc, kdesc, idesc2, on);
-        tc::mma_commit_if(&bars->empty[s], on);
+        if (code != kNoTile) {
+          const uint64_t kdesc = desc_plus(rdesc, (uint32_t)(s * G::kTileBytes));
+          const uint32_t dt = tmem + (uint32_t)(a * 256);
+          mma_tile_steps<D, 0, G::kKSteps>(code >= 0, RB, dt, qdesc, kdesc, idesc2, on);
+          tc::mma_commit_if(&bars->empty[s], on);
+        }
         tc::mma_commit_if(&bars->tfull[a], on);
         committed = it + 1;
+        if (code == kNoTile) break;
       }
     }
   } else if (warp < kEpiWarps) {
@@ -301,6 +361,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int sub = warp >> 2, quad = warp & 3;
     const float c = p.scale_log2;
     bool ok = true;
+    int it = 0;  // accumulators consumed so far (both passes)
 
     if (MODE & kPassStats) {
       // rows: row block wg, TMEM lane quadrant quad; keys: half `half` of each tile
@@ -310,19 +371,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int vis_end = min(rq.n, rq.p + w + 1);  // keys [0, vis_end) visible to the row
       float m_run = -INFINITY;
       float l_run = 0.f, l_comp = 0.f;  // compensated running sum of 2^(t - m_run)
-      for (int it = 0; it < n1; ++it) {
+      for (;; ++it) {
         const int a = it & 1;
         if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) {
           ok = false;
           break;
         }
         tc::tc_fence_after();
+        const int code = reinterpret_cast<volatile int*>(bars->accode)[a];
+        if (code < 0) break;  // a pass 2 tile or the end: pass 2 takes it from here
+        const int t = code;
         bool released = false;
         if (wg < RB) {
           const uint32_t taddr =
               tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(a * 256 + wg * 128 + half * 64);
-          const int key0 = info.j0 + it * kTileKeys + half * 64;
-          const bool all_vis = info.j0 + (it + 1) * kTileKeys <= rq.p;
+          const int key0 = t * kTileKeys + half * 64;
+          const bool all_vis = (t + 1) * kTileKeys <= rq.p;
           // this warp's 64 columns of the tile: two TMEM loads, one wait
           float v[64];
           __syncwarp();
@@ -432,24 +496,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = ok && tc::mbar_wait(&bars->gready, 0, abort, status) && !*abort;
       // merge every chunk of this (request, KV head) into -c_row
       if (ok) {
-        const int nch = (rq.n + p.chunk - 1) / p.chunk;
-        const size_t it0 = (size_t)rq.item0 + (size_t)info.g * nch;
-        for (int r = threadIdx.x; r < 256; r += kEpiWarps * 32) {
+        const size_t it0 = (size_t)rq.item0 + (size_t)info.g * info.nch;
+        // two threads per window row (adjacent lanes) fold alternate CTAs'
+        // partials in one pass (online rescaling, compensated sums), then
+        // combine through a shuffle in a fixed order
+        const int r = threadIdx.x >> 1, part = threadIdx.x & 1;
+        float m = -INFINITY, l = 0.f, comp = 0.f;
+        if (r < M) {
+#pragma unroll 4
+          for (int ch = part; ch < info.nch; ch += 2) {
+            const float2 pv = __ldcg(&partial[(it0 + ch) * M + r]);
+            if (pv.y > 0.f) {
+              if (pv.x > m) {
+                const float sc = exp2f(m - pv.x);
+                l *= sc;
+                comp *= sc;
+                m = pv.x;
+              }
+              const float term = pv.y * exp2f(pv.x - m) - comp;
+              const float tsum = l + term;
+              comp = (tsum - l) - term;
+              l = tsum;
+            }
+          }
+        }
+        const float mo = __shfl_xor_sync(0xffffffffu, m, 1);
+        const float lo = __shfl_xor_sync(0xffffffffu, l, 1);
+        if (part == 0) {
           float v = -INFINITY;
           if (r < M) {
-            float m = -INFINITY;
-            for (int ch = 0; ch < nch; ++ch) m = fmaxf(m, __ldcg(&partial[(it0 + ch) * M + r]).x);
-            float l = 0.f, comp = 0.f;  // compensated sum
-            for (int ch = 0; ch < nch; ++ch) {
-              const float2 pv = __ldcg(&partial[(it0 + ch) * M + r]);
-              if (pv.y > 0.f) {
-                const float term = pv.y * exp2f(pv.x - m) - comp;
-                const float t = l + term;
-                comp = (t - l) - term;
-                l = t;
-              }
-            }
-            v = -(m + log2f(l));
+            const float mm = fmaxf(m, mo);
+            const float ll = (l > 0.f ? l * exp2f(m - mm) : 0.f) + (lo > 0.f ? lo * exp2f(mo - mm) : 0.f);
+            v = -(mm + log2f(ll));
           }
           ncr[r] = v;
         }
@@ -463,12 +541,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       // keys: TMEM lane quadrant quad; window rows (columns): quarter `sub`
       const int key = quad * 32 + lane;  // TMEM lane = key within the tile
       float* out = scores + (size_t)info.g * p.score_rows + rq.score_off;
-      for (int it2 = 0; it2 < n2; ++it2) {
-        const int it = n1 + it2;
+      for (int it2 = 0;; ++it2, ++it) {
         const int a = it & 1;
-        const int t = n2 - 1 - it2;
         if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) break;
         tc::tc_fence_after();
+        const int code = reinterpret_cast<volatile int*>(bars->accode)[a];
+        if (code == kNoTile) break;  // the MMA warp has finished
+        const int t = -2 - code;
         const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(a * 256);
         float acc = 0.f;
         bool released = false;
@@ -484,30 +563,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
           released = true;
-          const int nv = c0 + 32 < NP ? 64 : 32;
-          // 2^(v c - c_row) in packed pairs; -c_row pairs come from shared memory
-          const uint64_t c2 = tc::pk2(c, c);
-          uint64_t a0 = 0, a1 = 0;
-#pragma unroll
-          for (int i = 0; i < 64; i += 4) {
-            if (i >= nv) break;
-            const float4 nc = *reinterpret_cast<const float4*>(ncr + c0 + i);
-            const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), c2, tc::pk2(nc.x, nc.y)));
-            const float2 y =
-                tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), c2, tc::pk2(nc.z, nc.w)));
-            float2 ex, ey;
-            if ((i & 31) < kMufuElems) {
-              ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
-              ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
-            } else {
-              ex = tc::exp2_poly2(x.x, x.y);
-              ey = tc::exp2_poly2(y.x, y.y);
-            }
-            a0 = tc::add2(a0, tc::pk2(ex.x, ex.y));
-            a1 = tc::add2(a1, tc::pk2(ey.x, ey.y));
-          }
-          const float2 s01 = tc::upk2(tc::add2(a0, a1));
-          acc = s01.x + s01.y;
+          // 2^(v c - c_row) over the columns the MMA wrote: NP - c0 is a
+          // multiple of 16, and columns past NP were never written
+          const int nv = min(64, NP - c0);
+          acc = nv == 64   ? vote_sum<64>(v, c, ncr + c0)
+                : nv == 48 ? vote_sum<48>(v, c, ncr + c0)
+                : nv == 32 ? vote_sum<32>(v, c, ncr + c0)
+                           : vote_sum<16>(v, c, ncr + c0);
         }
         if (!released) {
           tc::tc_fence_before();
@@ -515,21 +577,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
         }
         // combine the four quarters of the window rows through a double-buffered
-        // hand-off (bounded mbarrier waits, no named barrier); fixed sum order
+        // hand-off between the four warps of this lane quadrant (one SM
+        // sub-partition; bounded mbarrier waits, no named barrier); fixed sum order
         const int x = it2 & 1;
         const uint32_t xph = (uint32_t)((it2 >> 1) & 1);
         if (sub > 0) {
-          if (!tc::mbar_wait(&bars->xempty[x], xph ^ 1, abort, status)) break;
+          if (!tc::mbar_wait(&bars->xempty[x][quad], xph ^ 1, abort, status)) break;
           xbuf[(x * 3 + sub - 1) * 128 + key] = acc;
           __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->xfull[x]);
+          if (lane == 0) tc::mbar_arrive(&bars->xfull[x][quad]);
         } else {
-          if (!tc::mbar_wait(&bars->xfull[x], xph, abort, status)) break;
-          const int j = info.j0 + t * kTileKeys + key;
+          if (!tc::mbar_wait(&bars->xfull[x][quad], xph, abort, status)) break;
+          const int j = t * kTileKeys + key;
           const float* xb = xbuf + x * 3 * 128;
-          if (j < info.j1_pre) out[j] = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
+          if (j < rq.p) out[j] = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
           __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->xempty[x]);
+          if (lane == 0) tc::mbar_arrive(&bars->xempty[x][quad]);
         }
       }
     }
@@ -597,7 +660,7 @@ int coresident_ctas(const void* kernel, int smem, int slot) {
 template <int D>
 cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const CUtensorMap& tk,
                             float* scores, float2* partial, float* rowc, int32_t* status,
-                            cudaStream_t s) {
+                            int32_t* tilectr, cudaStream_t s) {
   using Gm = Geo<D>;
   uint32_t* gsync = reinterpret_cast<uint32_t*>(status) + kGridSyncWord;
   auto fused = ws_tc<D, kPassBoth>;
@@ -616,7 +679,7 @@ cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const 
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, fused, pt, tq, tk, partial, (const float*)rowc, scores, status,
-                           gsync);
+                           gsync, tilectr);
     count_launches(1);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
@@ -628,10 +691,12 @@ cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const 
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(votes, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
-  stats<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync);
+  stats<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync,
+                                              tilectr);
   e = launch_window_combine(pt, partial, rowc, s);
   if (e != cudaSuccess) return e;
-  votes<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync);
+  votes<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync,
+                                              tilectr);
   count_launches(2);
   return cudaGetLastError();
 }
@@ -680,15 +745,15 @@ EvictParams tc_item_params(const EvictParams& p) {
 
 cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, const void* K,
                                     float* scores, float2* partial, float* rowc, int32_t* status,
-                                    cudaStream_t s) {
+                                    int32_t* tilectr, cudaStream_t s) {
   const EvictParams pt = tc_item_params(p);
   CUtensorMap tq, tk;
   const uint64_t qrows = (uint64_t)p.batch * p.hq * p.window;
   const uint64_t krows = (uint64_t)p.hkv * p.kv_rows;
   if (!make_bf16_map(&tq, q_win, p.d, qrows, 128) || !make_bf16_map(&tk, K, p.d, krows, 128))
     return cudaErrorInvalidValue;
-  return p.d == 64 ? launch_tc_typed<64>(pt, tq, tk, scores, partial, rowc, status, s)
-                   : launch_tc_typed<128>(pt, tq, tk, scores, partial, rowc, status, s);
+  return p.d == 64 ? launch_tc_typed<64>(pt, tq, tk, scores, partial, rowc, status, tilectr, s)
+                   : launch_tc_typed<128>(pt, tq, tk, scores, partial, rowc, status, tilectr, s);
 }
 
 }  // namespace tb

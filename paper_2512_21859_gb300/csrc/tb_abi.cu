@@ -123,6 +123,9 @@ EvictWorkspace carve_evict(const EvictParams& p) {
   size_t off = 0;
   w.status = off;
   off += kStatusBytes;
+  w.tilectr = off;
+  off = align_up(off + 2 * sizeof(int32_t) * (size_t)p.batch * p.hkv, 256);
+  w.zeroed = off;
   w.scores = off;
   off = align_up(off + sizeof(float) * (size_t)p.hkv * p.score_rows, 256);
   w.partial = off;
@@ -217,7 +220,8 @@ T* at(void* base, size_t off) {
 tb_status run_window_scores(const EvictParams& p, const EvictWorkspace& w, const void* q_win,
                             const void* K, float* scores, void* ws, cudaStream_t s) {
   return cuda_status(launch_window_scores(p, q_win, K, scores, at<float2>(ws, w.partial),
-                                          at<float>(ws, w.rowc), at<int32_t>(ws, w.status), s));
+                                          at<float>(ws, w.rowc), at<int32_t>(ws, w.status),
+                                          at<int32_t>(ws, w.tilectr), s));
 }
 
 tb_status run_select(const EvictParams& p, const EvictWorkspace& w, const float* scores,
@@ -235,9 +239,9 @@ void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order
 
 cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
                                  float* scores, float2* partial, float* rowc, int32_t* status,
-                                 cudaStream_t s) {
+                                 int32_t* tilectr, cudaStream_t s) {
   if (window_scores_tc_supported(p))
-    return launch_window_scores_tc(p, q_win, K, scores, partial, rowc, status, s);
+    return launch_window_scores_tc(p, q_win, K, scores, partial, rowc, status, tilectr, s);
   return launch_window_scores_simt(p, q_win, K, scores, partial, rowc, s);
 }
 
@@ -304,7 +308,7 @@ tb_status tb_window_scores(const tb_evict_desc* desc, const void* q_win, const v
   const EvictWorkspace w = carve_evict(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, w.zeroed, s))) != TB_OK) return st;
   return run_window_scores(p, w, q_win, K, scores, workspace, s);
 }
 
@@ -319,7 +323,7 @@ tb_status tb_select_topk(const tb_evict_desc* desc, const float* scores, int32_t
   const EvictWorkspace w = carve_evict(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, w.zeroed, s))) != TB_OK) return st;
   return run_select(p, w, scores, idx, pooled, workspace, s);
 }
 
@@ -348,7 +352,7 @@ tb_status tb_score_evict(const tb_evict_desc* desc, const void* q_win, const voi
   const EvictWorkspace w = carve_evict(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, kStatusBytes, s))) != TB_OK) return st;
+  if ((st = cuda_status(cudaMemsetAsync(workspace, 0, w.zeroed, s))) != TB_OK) return st;
   float* scores = at<float>(workspace, w.scores);
   if ((st = run_window_scores(p, w, q_win, K, scores, workspace, s)) != TB_OK) return st;
   if ((st = run_select(p, w, scores, idx, pooled, workspace, s)) != TB_OK) return st;

@@ -77,8 +77,10 @@ DecodeWorkspace carve_decode(const DecodeParams& p);
 tb_status cuda_status(cudaError_t e);
 
 // Workspace carving for the eviction calls (byte offsets, 256-aligned).
+// status: kStatusBytes; tilectr: two tile counters per (request, KV head) of
+// the tensor-core scoring kernel; [0, zeroed) is cleared by every call.
 struct EvictWorkspace {
-  size_t status, scores, partial, rowc, pooled, total;
+  size_t status, tilectr, zeroed, scores, partial, rowc, pooled, total;
 };
 
 // 2-D bf16 TMA map over rows of d elements, boxes of box_rows x 64 columns
@@ -93,7 +95,7 @@ void count_launches(int n);
 // ---------------------------------------------------------------------------
 cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
                                  float* scores, float2* partial, float* rowc,
-                                 int32_t* status, cudaStream_t s);
+                                 int32_t* status, int32_t* tilectr, cudaStream_t s);
 cudaError_t launch_window_scores_simt(const EvictParams& p, const void* q_win, const void* K,
                                       float* scores, float2* partial, float* rowc,
                                       cudaStream_t s);
@@ -104,7 +106,7 @@ cudaError_t launch_window_combine(const EvictParams& p, const float2* partial, f
 bool window_scores_tc_supported(const EvictParams& p);
 cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, const void* K,
                                     float* scores, float2* partial, float* rowc, int32_t* status,
-                                    cudaStream_t s);
+                                    int32_t* tilectr, cudaStream_t s);
 cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled,
                         cudaStream_t s);
 cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* idx,
