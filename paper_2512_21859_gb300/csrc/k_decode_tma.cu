@@ -47,7 +47,9 @@ struct DGeo {
   // (rows padded by 8 floats so the fragment stores hit distinct banks)
   static constexpr int kDS = D + 8;
   static constexpr int kMergeO = kWarps * 16 * kDS * 4;
-  static_assert(kMergeO + kWarps * 16 * 8 <= kRing, "merge area must fit in the ring");
+  // O, (m, l) per warp, then the per-head warp weights [16][kWarps]
+  static_assert(kMergeO + kWarps * 16 * 8 + 16 * kWarps * 4 <= kRing,
+                "merge area must fit in the ring");
   static constexpr int kMaxSplits = kRing / (16 * 4);  // weights table [G <= 16][splits]
   static constexpr int kBarOff = kRing;
   static constexpr int kSmem = kBarOff + 64 + 1024;  // + alignment slack
@@ -339,25 +341,38 @@ __global__ void __launch_bounds__(kThreads, 1)
     mml[(warp * 16 + r0 + 8) * 2 + 1] = l_run[1];
   }
   __syncthreads();
-  for (int e = tid; e < G * D; e += kThreads) {
-    const int h = e / D, dim = e % D;
+  // per head: the warps' weights 2^(m_w - M) (thread h), then every output
+  // element as one pass of independent loads over the warps
+  float* wgt = mml + kWarps * 16 * 2;  // [G][kWarps]
+  if (tid < G) {
+    const int h = tid;
     float M = -INFINITY;
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mml[(w * 16 + h) * 2]);
-    float L = 0.f, O = 0.f;
-    if (M != -INFINITY) {
+    float L = 0.f;
 #pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        const float mw = mml[(w * 16 + h) * 2];
-        if (mw != -INFINITY) {
-          const float wt = fast_exp2(mw - M);
-          L = fmaf(mml[(w * 16 + h) * 2 + 1], wt, L);
-          O = fmaf(mo[(w * 16 + h) * DS + dim], wt, O);
-        }
-      }
+    for (int w = 0; w < kWarps; ++w) {
+      const float mw = mml[(w * 16 + h) * 2];
+      const float wt = (M != -INFINITY && mw != -INFINITY) ? fast_exp2(mw - M) : 0.f;
+      wgt[h * kWarps + w] = wt;
+      L = fmaf(mml[(w * 16 + h) * 2 + 1], wt, L);
     }
-    part_o[(part_base + (size_t)h * p.splits) * D + dim] = O;
-    if (dim == 0) part_ml[part_base + (size_t)h * p.splits] = make_float2(M, L);
+    part_ml[part_base + (size_t)h * p.splits] = make_float2(M, L);
+  }
+  __syncthreads();
+  for (int e = tid; e < G * (D / 4); e += kThreads) {
+    const int h = e / (D / 4), d4 = e % (D / 4);
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const float wt = wgt[h * kWarps + w];
+      const float4 ow = *reinterpret_cast<const float4*>(mo + (w * 16 + h) * DS + 4 * d4);
+      O.x = fmaf(ow.x, wt, O.x);
+      O.y = fmaf(ow.y, wt, O.y);
+      O.z = fmaf(ow.z, wt, O.z);
+      O.w = fmaf(ow.w, wt, O.w);
+    }
+    *reinterpret_cast<float4*>(part_o + (part_base + (size_t)h * p.splits) * D + 4 * d4) = O;
   }
 
   // ---- the last split CTA of this (request, KV head) merges every split
@@ -395,7 +410,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const size_t hb = head0 + (size_t)h * p.splits;
     const float* wh = wts + h * p.splits;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
+#pragma unroll 16
     for (int sp = 0; sp < p.splits; ++sp) {
       const float wgt = wh[sp];
       const float4 ov = __ldcg(reinterpret_cast<const float4*>(part_o + (hb + sp) * D) + d4);
