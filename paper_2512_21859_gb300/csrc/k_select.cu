@@ -374,8 +374,11 @@ bool select_cluster_supported(const EvictParams& p) {
   return slice <= kClusterSliceMax;
 }
 
+// One CTA per 4096 keys of the longest prefix, up to 8 (the portable cluster
+// size): the kernel is bound by the latency of its phases, and on GB300 the
+// smaller slices measured faster (32K keys: 23.6 -> 20.8 us with 8 CTAs).
 int select_cluster_size(const EvictParams& p) {
-  int cs = (p.max_p + 8191) / 8192;
+  int cs = (p.max_p + 4095) / 4096;
   return cs < 1 ? 1 : (cs > 8 ? 8 : cs);
 }
 
