@@ -205,13 +205,25 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   __syncthreads();
   constexpr int kMaxPer = kClusterSliceMax / kCsThreads;
   unsigned reg[kMaxPer];
+  if (half == 3) {  // pool_k = 7: the window as compile-time loads
 #pragma unroll
-  for (int r = 0; r < kMaxPer; ++r) {
-    const int i = tid + r * kCsThreads;
-    if (i < cnt) {
-      float m = keys_f[i];
-      for (int t = 1; t <= 2 * half; ++t) m = fmaxf(m, keys_f[i + t]);
-      reg[r] = __float_as_uint(m);
+    for (int r = 0; r < kMaxPer; ++r) {
+      const int i = tid + r * kCsThreads;
+      if (i < cnt) {
+        const float* x = keys_f + i;
+        reg[r] = __float_as_uint(fmaxf(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])),
+                                       fmaxf(fmaxf(x[4], x[5]), x[6])));
+      }
+    }
+  } else {
+#pragma unroll
+    for (int r = 0; r < kMaxPer; ++r) {
+      const int i = tid + r * kCsThreads;
+      if (i < cnt) {
+        float m = keys_f[i];
+        for (int t = 1; t <= 2 * half; ++t) m = fmaxf(m, keys_f[i + t]);
+        reg[r] = __float_as_uint(m);
+      }
     }
   }
   __syncthreads();
@@ -238,14 +250,19 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
       unsigned* h = sh.hist[pass & 1];
       for (int t = tid; t < 256; t += kCsThreads) h[t] = 0;
       __syncthreads();
-      for (int i = tid; i - lane < cnt; i += kCsThreads) {
-        const bool valid = i < cnt && ((keys[i < cnt ? i : 0] & mask) == prefix);
-        const unsigned dg = valid ? (keys[i] >> shift) & 255u : 256u;
-        const unsigned d0 = __shfl_sync(0xffffffffu, dg, 0);
-        if (__all_sync(0xffffffffu, dg == d0)) {
-          if (lane == 0 && d0 < 256u) atomicAdd(&h[d0], 32u);
-        } else if (valid) {
-          atomicAdd(&h[dg], 1u);
+      // four keys per round: their loads and digits are independent (the
+      // kernel is bound by the latency of these loops, not by throughput)
+      for (int i0 = tid; i0 < cnt; i0 += 4 * kCsThreads) {
+        unsigned kv[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int i = i0 + q * kCsThreads;
+          kv[q] = i < cnt ? keys[i] : 0u;
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int i = i0 + q * kCsThreads;
+          if (i < cnt && (kv[q] & mask) == prefix) atomicAdd(&h[(kv[q] >> shift) & 255u], 1u);
         }
       }
       cluster.sync();
@@ -297,11 +314,19 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   const int wlo = min(cnt, warp * run), whi = min(cnt, wlo + run);
   int gt_w = 0, eq_w = 0;
   if (k > 0) {
-    for (int base = wlo; base < whi; base += 32) {
-      const int i = base + lane;
-      const unsigned u = i < whi ? keys[i] : 0u;
-      gt_w += __popc(__ballot_sync(0xffffffffu, i < whi && u > tau));
-      eq_w += __popc(__ballot_sync(0xffffffffu, i < whi && u == tau));
+    for (int b0 = wlo; b0 < whi; b0 += 128) {
+      unsigned kv[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int i = b0 + 32 * q + lane;
+        kv[q] = i < whi ? keys[i] : 0u;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int i = b0 + 32 * q + lane;
+        gt_w += __popc(__ballot_sync(0xffffffffu, i < whi && kv[q] > tau));
+        eq_w += __popc(__ballot_sync(0xffffffffu, i < whi && kv[q] == tau));
+      }
     }
   }
   if (lane == 0) {
@@ -333,18 +358,26 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   }
   if (k > 0) {
     const unsigned lt = (1u << lane) - 1u;
-    for (int base = wlo; base < whi; base += 32) {
-      const int i = base + lane;
-      const unsigned u = i < whi ? keys[i] : 0u;
-      const bool gt = i < whi && u > tau;
-      const bool eq = i < whi && u == tau;
-      const unsigned em = __ballot_sync(0xffffffffu, eq);
-      const bool sel = gt || (eq && eqbase + __popc(em & lt) < need);
-      const unsigned sm = __ballot_sync(0xffffffffu, sel);
-      const int pos = selbase + __popc(sm & lt);
-      if (sel && pos < k) out[pos] = lo + i;
-      selbase += __popc(sm);
-      eqbase += __popc(em);
+    for (int b0 = wlo; b0 < whi; b0 += 128) {
+      unsigned kv[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int i = b0 + 32 * q + lane;
+        kv[q] = i < whi ? keys[i] : 0u;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int i = b0 + 32 * q + lane;
+        const bool gt = i < whi && kv[q] > tau;
+        const bool eq = i < whi && kv[q] == tau;
+        const unsigned em = __ballot_sync(0xffffffffu, eq);
+        const bool sel = gt || (eq && eqbase + __popc(em & lt) < need);
+        const unsigned sm = __ballot_sync(0xffffffffu, sel);
+        const int pos = selbase + __popc(sm & lt);
+        if (sel && pos < k) out[pos] = lo + i;
+        selbase += __popc(sm);
+        eqbase += __popc(em);
+      }
     }
   }
   cluster.sync();  // no CTA leaves while another may still read its shared memory
