@@ -169,6 +169,7 @@ struct ClusterSelectShared {
   unsigned total[256];
   int wgt[kCsWarps], weq[kCsWarps];
   int cta_cnt[2];  // this CTA's (greater, equal) counts, read by the cluster
+  int rank_cnt[8][2];  // the lower ranks' counts (cluster size <= 8)
   unsigned prefix;
   int need;
 };
@@ -197,10 +198,21 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   if (rank == 0)
     for (int t = tid; t < p.window; t += kCsThreads) out[k + t] = P + t;
 
-  // slice + halo, -inf outside the prefix (scores are >= 0, so max is exact)
-  for (int i = tid; i < cnt + 2 * half; i += kCsThreads) {
-    const int j = lo - half + i;
-    keys_f[i] = (j >= 0 && j < P) ? S[j] : -INFINITY;
+  // slice + halo, -inf outside the prefix (scores are >= 0, so max is exact);
+  // four loads in flight per thread
+  const int nin = cnt + 2 * half;
+  for (int i0 = tid; i0 < nin; i0 += 4 * kCsThreads) {
+    float x[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * kCsThreads, j = lo - half + i;
+      x[q] = (i < nin && j >= 0 && j < P) ? S[j] : -INFINITY;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * kCsThreads;
+      if (i < nin) keys_f[i] = x[q];
+    }
   }
   __syncthreads();
   constexpr int kMaxPer = kClusterSliceMax / kCsThreads;
@@ -334,21 +346,31 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
     sh.weq[warp] = eq_w;
   }
   __syncthreads();
-  if (tid == 0) {
-    int gsum = 0, esum = 0;
-    for (int w = 0; w < kCsWarps; ++w) {
-      gsum += sh.wgt[w];
-      esum += sh.weq[w];
+  if (warp == 0) {
+    int gsum = sh.wgt[lane], esum = sh.weq[lane];
+    for (int off = 16; off > 0; off >>= 1) {
+      gsum += __shfl_xor_sync(0xffffffffu, gsum, off);
+      esum += __shfl_xor_sync(0xffffffffu, esum, off);
     }
-    sh.cta_cnt[0] = gsum;
-    sh.cta_cnt[1] = esum;
+    if (lane == 0) {
+      sh.cta_cnt[0] = gsum;
+      sh.cta_cnt[1] = esum;
+    }
   }
   cluster.sync();
+  // the lower ranks' counts, all remote loads at once
+  if (tid < 16) {
+    const int r = tid >> 1;
+    sh.rank_cnt[r][tid & 1] = r < rank ? cluster.map_shared_rank(sh.cta_cnt, r)[tid & 1] : 0;
+  }
+  __syncthreads();
+  // no shared memory of another CTA is read after this point: arrive now, and
+  // wait (so that none leaves while another may still read it) at the end
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
   // offsets of this CTA: ties are kept in index order until `need` are in
   int eqbase = 0, selbase = 0;
   for (int r = 0; r < rank; ++r) {
-    const int* c = cluster.map_shared_rank(sh.cta_cnt, r);
-    const int tg = c[0], te = c[1];
+    const int tg = sh.rank_cnt[r][0], te = sh.rank_cnt[r][1];
     selbase += tg + max(0, min(need - eqbase, te));
     eqbase += te;
   }
@@ -380,7 +402,7 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
       }
     }
   }
-  cluster.sync();  // no CTA leaves while another may still read its shared memory
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 }  // namespace
