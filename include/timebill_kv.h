@@ -205,7 +205,9 @@ tb_status tb_decode_attn(const tb_decode_desc *desc, const void *q,
  * workspace used by the calls above: TB_OK, TB_ERR_TIMEOUT (a bounded
  * device-side wait gave up) or TB_ERR_INVALID_ARG (a device-side range check
  * fired, e.g. a decode length above its cap). *raw (if not NULL) receives the
- * word itself. The word is cleared at the start of every call.
+ * word itself. The word is cleared at the start of every call that can set
+ * it: tb_window_scores, tb_score_evict and tb_decode_attn (tb_select_topk
+ * and tb_gather_kv never set it and leave it as it was).
  */
 tb_status tb_read_status(const void *workspace, size_t workspace_bytes,
                          tb_stream_t stream, int32_t *raw);
