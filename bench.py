@@ -109,6 +109,21 @@ def dist_init(world, use_cuda):
     return dist
 
 
+def max_over_ranks(dist, value, device=None):
+    """The largest of every rank's `value`: the job's time is its slowest rank's."""
+    if not dist:
+        return float(value)
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(world, step_bytes, steps, total_ms):
+    """Whole-job GB/s: every rank moved step_bytes per step (weak scaling)."""
+    return world * step_bytes * steps / (total_ms * 1e-3) / 1e9
+
+
 # ---------------------------------------------------------------------------
 # clocks sampled during the timed region
 # ---------------------------------------------------------------------------
@@ -323,16 +338,13 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     torch.cuda.synchronize(dev)
     clocks = sampler.stop()
     launches = kernels_per_step * K
-    if dist:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(dist, total_ms, dev)
     for d in layers:
         st, raw = tb.tb_read_status(d["dws"], stream=stream)
         assert st == tb.TB_OK, raw
     stage_ms = {s: sum(ev[j].elapsed_time(ev[j + 1]) for ev in evs) / K for j, s in enumerate(stages)}
     ms_step = total_ms / K
-    value = world * ab["step"] * K / (total_ms * 1e-3) / 1e9
+    value = job_value(world, ab["step"], K, total_ms)
 
     # roofline of the dominant stage
     with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
