@@ -249,6 +249,50 @@ tb_status tb_decode_attn_noalloc(const tb_decode_desc *desc, const void *q,
                                  const int32_t *lens, void *out,
                                  tb_stream_t stream);
 
+/*
+ * Execution-time model of "Profiling-based Fitting" (Eq. 6a and 6b), in
+ * seconds: the prefill of N_x prompt tokens takes a N_x^2 + b N_x + c, one
+ * decoding step over N_kv cached tokens takes p N_kv + q. Host memory.
+ */
+typedef struct {
+  double a, b, c;
+  double p, q;
+} tb_time_model;
+
+/*
+ * Eq. 12: the worst-case execution time estimate of one request, in seconds:
+ * the prefill of n_x tokens plus the decoding steps i = 1 .. n_w - 1, step i
+ * over (1 - alpha) n_x + i - 1 cached tokens (Eqs. 9-11). n_w is the
+ * pessimistic response length (tb_alpha_star reports the one it uses). Host
+ * only; no device work.
+ * Errors: TB_ERR_INVALID_ARG for a NULL pointer, n_x < 1, n_w < 1, alpha
+ * outside [0, 1] or a non-finite coefficient.
+ */
+tb_status tb_wcet(const tb_time_model *model, int64_t n_x, double alpha,
+                  int64_t n_w, double *t_out);
+
+/*
+ * The eviction ratio a time budget allows (Prob. 13 of "Time-Budgeted LLM
+ * Inference Mechanism", closed form Eq. 14): the smallest alpha in
+ * [0, alpha_max] with t_predict + WCET(alpha) <= budget, assuming the
+ * pessimistic response length N_W = min(ceil(k * n_hat), n_max) (at least 1)
+ * from the predicted length n_hat and the pessimistic factor k. When no alpha
+ * in the range fits, alpha_max (the caller's overrun policy takes over).
+ * In closed form, with n = N_W - 1 decoding steps:
+ *   alpha = 1 - (budget - t_prefill - t_predict) / (p N_x n)
+ *             + (n - 1) / (2 N_x) + q / (p N_x),   clamped to [0, alpha_max].
+ * (The sum of Eq. 11 gives the middle term without p; the paper prints it
+ * over 2 p N_x. The lower clamp is the alpha >= 0 constraint of Prob. 13.)
+ * Writes *alpha_out and, if n_w_out is not NULL, N_W. Host only.
+ * Errors: TB_ERR_INVALID_ARG for a NULL model or alpha_out, n_x < 1,
+ * n_max < 1, n_hat < 0, k < 1, alpha_max outside [0, 1), p <= 0 or a
+ * non-finite input.
+ */
+tb_status tb_alpha_star(const tb_time_model *model, int64_t n_x, double n_hat,
+                        double k, int64_t n_max, double t_predict,
+                        double budget, double alpha_max, double *alpha_out,
+                        int64_t *n_w_out);
+
 #ifdef __cplusplus
 }
 #endif

@@ -26,6 +26,10 @@ from the exact input values):
 6. The compact cache: bit copies of those K and V rows.
 7. Decode-step attention (Eq. 8's N_kv^i keys, attention definition): one
    query per head over the first ``len`` rows of the compact cache.
+8. The eviction ratio the time budget allows (Prob. 13 of "Time-Budgeted LLM
+   Inference Mechanism"): the smallest alpha in [0, alpha_max] whose
+   worst-case execution time estimate (Eq. 12, built from Eqs. 6a, 9-11)
+   fits the budget, found here from its definition by bisection.
 
 Parity status: every function here is pinned by tests/test_oracle_pins.py
 (hand-derived closed forms, brute force, invariants, library routines).
@@ -46,6 +50,9 @@ __all__ = [
     "score_evict",
     "decode_attention",
     "decode_batch",
+    "pessimistic_length",
+    "wcet",
+    "alpha_star",
 ]
 
 
@@ -198,3 +205,53 @@ def decode_batch(q: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, lens: Sequence[i
         off, L = int(cache_offset[b]), int(lens[b])
         out[b] = decode_attention(q[b], Kc[:, off:off + L], Vc[:, off:off + L], L)
     return out
+
+
+# ---------------------------------------------------------------------------
+# step 8: the eviction ratio a time budget allows
+# ---------------------------------------------------------------------------
+
+def pessimistic_length(n_hat: float, k: float, n_max: int) -> int:
+    """N_W = min(k N_hat, N_max) (Section "End-to-end Execution Time
+    Prediction"). Reading: k N_hat is rounded up, the pessimistic side, since
+    it counts decoding steps."""
+    return int(min(math.ceil(k * n_hat), n_max))
+
+
+def wcet(a: float, b: float, c: float, p: float, q: float, n_x: int, alpha: float,
+         n_w: int) -> float:
+    """Eq. 12: the prefill time of Eq. 6a plus the decoding phase of Eq. 11,
+    the sum over steps i = 1 .. N_W - 1 of Eq. 10, p ((1 - alpha) N_x + i - 1) + q.
+    The sum is taken term by term."""
+    t_prefill = a * n_x * n_x + b * n_x + c
+    t_decode = 0.0
+    for i in range(1, n_w):
+        t_decode += p * ((1.0 - alpha) * n_x + i - 1) + q
+    return t_prefill + t_decode
+
+
+def alpha_star(a: float, b: float, c: float, p: float, q: float, n_x: int, n_hat: float,
+               k: float, n_max: int, t_predict: float, budget: float,
+               alpha_max: float) -> float:
+    """Prob. 13: minimise alpha subject to t_Predict + WCET(alpha) <= T and
+    0 <= alpha <= alpha_max. WCET is non-increasing in alpha (p > 0), so the
+    smallest feasible alpha is found by bisection on the constraint itself.
+    When no alpha in range meets the budget, alpha_max (the most the budget
+    can be helped; the paper's overrun strategies take it from there)."""
+    n_w = pessimistic_length(n_hat, k, n_max)
+
+    def excess(al: float) -> float:
+        return t_predict + wcet(a, b, c, p, q, n_x, al, n_w) - budget
+
+    if excess(0.0) <= 0.0:
+        return 0.0
+    if excess(alpha_max) > 0.0:
+        return float(alpha_max)
+    lo, hi = 0.0, float(alpha_max)  # excess(lo) > 0 >= excess(hi)
+    for _ in range(80):
+        mid = 0.5 * (lo + hi)
+        if excess(mid) <= 0.0:
+            hi = mid
+        else:
+            lo = mid
+    return hi

@@ -24,6 +24,7 @@ __all__ = [
     "tb_window_scores", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
     "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_exp2",
+    "TimeModel", "tb_wcet", "tb_alpha_star",
 ]
 
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
@@ -103,6 +104,10 @@ def load():
         "tb_read_status": (I, [P, SZ, P, ctypes.POINTER(I)]),
         "tb_decode_attn_noalloc": (I, [P, P, P, P, P, P, P]),
         "tb_diag_exp2": (I, [P, P, ctypes.c_int64, P]),
+        "tb_wcet": (I, [P, ctypes.c_int64, ctypes.c_double, ctypes.c_int64, ctypes.POINTER(ctypes.c_double)]),
+        "tb_alpha_star": (I, [P, ctypes.c_int64, ctypes.c_double, ctypes.c_double, ctypes.c_int64,
+                              ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                              ctypes.POINTER(ctypes.c_double), _I64P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -146,6 +151,12 @@ def _stream(stream) -> Optional[int]:
 def _check(status: int, where: str):
     if status != TB_OK:
         raise TbError(status, where)
+
+
+class TimeModel(ctypes.Structure):
+    """tb_time_model: prefill a N^2 + b N + c and decode step p N_kv + q, seconds."""
+    _fields_ = [("a", ctypes.c_double), ("b", ctypes.c_double), ("c", ctypes.c_double),
+                ("p", ctypes.c_double), ("q", ctypes.c_double)]
 
 
 class EvictDesc:
@@ -318,3 +329,21 @@ def tb_read_status(workspace, workspace_bytes=None, stream=None):
     if st not in (TB_OK, TB_ERR_TIMEOUT, TB_ERR_INVALID_ARG):
         raise TbError(st, "tb_read_status")
     return st, raw.value
+
+
+def tb_wcet(model: TimeModel, n_x: int, alpha: float, n_w: int) -> float:
+    t = ctypes.c_double()
+    _check(load().tb_wcet(ctypes.byref(model), int(n_x), float(alpha), int(n_w), ctypes.byref(t)),
+           "tb_wcet")
+    return t.value
+
+
+def tb_alpha_star(model: TimeModel, n_x: int, n_hat: float, k: float, n_max: int,
+                  t_predict: float, budget: float, alpha_max: float):
+    """(alpha*, N_W) of the time budget (host computation)."""
+    a = ctypes.c_double()
+    n_w = ctypes.c_int64()
+    _check(load().tb_alpha_star(ctypes.byref(model), int(n_x), float(n_hat), float(k), int(n_max),
+                                float(t_predict), float(budget), float(alpha_max), ctypes.byref(a),
+                                ctypes.byref(n_w)), "tb_alpha_star")
+    return a.value, n_w.value

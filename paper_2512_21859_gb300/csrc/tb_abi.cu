@@ -3,6 +3,8 @@
 // Every check runs on the host before the first CUDA call, so an invalid
 // call returns without touching the GPU or any output buffer.
 #include <cuda_runtime.h>
+
+#include <cmath>
 #include <math.h>
 #include <string.h>
 
@@ -276,6 +278,58 @@ tb_status tb_retained_count(int64_t n, int32_t window, double alpha, int64_t* k_
   if (!retained(n, window, alpha, &k, &r)) return TB_ERR_INVALID_ARG;
   *k_out = k;
   *r_out = r;
+  return TB_OK;
+}
+
+namespace {
+
+bool model_ok(const tb_time_model* m) {
+  return m && std::isfinite(m->a) && std::isfinite(m->b) && std::isfinite(m->c) &&
+         std::isfinite(m->p) && std::isfinite(m->q);
+}
+
+double prefill_time(const tb_time_model* m, double nx) { return (m->a * nx + m->b) * nx + m->c; }
+
+}  // namespace
+
+// Eq. 12 with the decoding-phase sum of Eq. 11 in closed form:
+// sum_{i=1..n} p((1 - alpha) N_x + i - 1) + q = n p (1 - alpha) N_x + p n (n - 1) / 2 + n q.
+tb_status tb_wcet(const tb_time_model* model, int64_t n_x, double alpha, int64_t n_w,
+                  double* t_out) {
+  if (!model_ok(model) || !t_out || n_x < 1 || n_w < 1 || !(alpha >= 0.0 && alpha <= 1.0))
+    return TB_ERR_INVALID_ARG;
+  const double nx = (double)n_x, n = (double)(n_w - 1);
+  *t_out = prefill_time(model, nx) + n * model->p * (1.0 - alpha) * nx +
+           model->p * n * (n - 1.0) / 2.0 + n * model->q;
+  return TB_OK;
+}
+
+// Prob. 13 through the closed form of Eq. 14 (with the middle term as the
+// sum of Eq. 11 gives it, and the alpha >= 0 clamp): the constraint
+// t_predict + WCET(alpha) <= budget is linear in alpha with slope -p N_x n.
+tb_status tb_alpha_star(const tb_time_model* model, int64_t n_x, double n_hat, double k,
+                        int64_t n_max, double t_predict, double budget, double alpha_max,
+                        double* alpha_out, int64_t* n_w_out) {
+  if (!model_ok(model) || !alpha_out || n_x < 1 || n_max < 1 || !(n_hat >= 0.0) ||
+      !std::isfinite(n_hat) || !(k >= 1.0) || !std::isfinite(k) || !(model->p > 0.0) ||
+      !(alpha_max >= 0.0 && alpha_max < 1.0) || !std::isfinite(t_predict) ||
+      !std::isfinite(budget))
+    return TB_ERR_INVALID_ARG;
+  const double kn = std::ceil(k * n_hat);
+  int64_t n_w = kn >= (double)n_max ? n_max : (int64_t)kn;
+  if (n_w < 1) n_w = 1;
+  const double nx = (double)n_x, n = (double)(n_w - 1);
+  const double slack = budget - prefill_time(model, nx) - t_predict;
+  double alpha;
+  if (n_w == 1) {
+    alpha = slack >= 0.0 ? 0.0 : alpha_max;  // no decoding step: alpha cannot help
+  } else {
+    const double req = 1.0 - slack / (model->p * nx * n) + (n - 1.0) / (2.0 * nx) +
+                       model->q / (model->p * nx);
+    alpha = std::fmin(alpha_max, std::fmax(0.0, req));
+  }
+  *alpha_out = alpha;
+  if (n_w_out) *n_w_out = n_w;
   return TB_OK;
 }
 

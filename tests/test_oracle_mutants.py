@@ -31,6 +31,11 @@ MUTANTS = {
     "budget counts the window inside": ("return k, k + window", "return max(k - window, 0), max(k - window, 0) + window"),
     "decode scale dropped": ("s = sigma * (kk @ q[h])", "s = kk @ q[h]"),
     "decode attends one row too many": ("kk = np.asarray(Kc[g, :length]", "kk = np.asarray(Kc[g, :length + 1]"),
+    "decoding steps counted from i = 0": ("for i in range(1, n_w):", "for i in range(0, n_w):"),
+    "decode step over N_kv without the eviction": ("p * ((1.0 - alpha) * n_x + i - 1) + q", "p * (n_x + i - 1) + q"),
+    "per-step constant dropped": ("t_decode += p * ((1.0 - alpha) * n_x + i - 1) + q", "t_decode += p * ((1.0 - alpha) * n_x + i - 1)"),
+    "pessimistic length rounded down": ("int(min(math.ceil(k * n_hat), n_max))", "int(min(math.floor(k * n_hat), n_max))"),
+    "predictor overhead ignored": ("return t_predict + wcet(a, b, c, p, q, n_x, al, n_w) - budget", "return wcet(a, b, c, p, q, n_x, al, n_w) - budget"),
 }
 
 
@@ -80,6 +85,11 @@ def _pins_pass(m):
         out = m.decode_attention(qq[:1, 0], KK, VV, 20)
         ref = bf.attention(qq[0, 0].tolist(), KK[0].tolist(), VV[0].tolist(), 20)
         if not np.allclose(out[0], ref, rtol=1e-12):
+            return False
+        # the budgeted eviction ratio: the hand example of tests/test_alpha_star.py
+        al = m.alpha_star(1e-9, 2e-6, 1e-4, 1e-6, 5e-5, 1000, 10, 1.0, 100, 3e-4, 8e-3, 0.95)
+        want = 1.0 - (8e-3 - 3e-4 - (1e-3 + 2e-3 + 1e-4) - 9 * 5e-5 - 36e-6) / 9e-3
+        if abs(al - want) > 1e-12 or m.pessimistic_length(10, 1.25, 100) != 13:
             return False
         return True
     except (ValueError, IndexError, AssertionError):
