@@ -90,6 +90,27 @@ def alg_bytes(wl, n, alpha, lens):
             "decode_attn": decode, "evict": evict_min, "step": evict_min + decode, "R": R}
 
 
+def stage_rooflines(wl, n, ab, stage_ms, peaks):
+    """Every stage against its roofline: algorithmic bytes over the stage time
+    against the measured copy bandwidth; the window scoring also as a tensor
+    contraction (2 Hq W d flops per key and pass, two passes) against the
+    measured sustained bf16 rate (its kernel runs inside a long step)."""
+    hbm = float(peaks["hbm_gbs"])
+    out = {}
+    for s, ms in stage_ms.items():
+        gbs = ab[s] / (ms * 1e-3) / 1e9
+        out[s] = {"bound": "hbm", "alg_bytes": int(ab[s]), "us": round(1e3 * ms, 2),
+                  "achieved_gbs": round(gbs, 1), "frac": round(gbs / hbm, 4)}
+    if "window_scores" in stage_ms and wl.dtype == "bf16":
+        flops = 2 * (2.0 * wl.hq * wl.window * wl.head_dim * float(np.sum(n)))
+        tf = flops / (stage_ms["window_scores"] * 1e-3) / 1e12
+        peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+        out["window_scores"]["tensor"] = {"flops": flops, "achieved_tflops": round(tf, 1),
+                                          "peak_tflops": peak, "frac": round(tf / peak, 4),
+                                          "peak_source": "measured sustained bf16 (MEASURED_PEAKS.json)"}
+    return out
+
+
 # ---------------------------------------------------------------------------
 # distributed plumbing
 # ---------------------------------------------------------------------------
@@ -378,6 +399,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                 "decode": round(ab["decode_attn"] / (stage_ms["decode_attn"] * 1e-3) / 1e9, 1)},
         "frac_of_8tbs": round(value / world / NOMINAL_HBM_GBS, 4),
         "roofline": roof,
+        "stage_roofline": stage_rooflines(wl, n, ab, stage_ms, peaks),
         "e2e": e2e,
         "gpu_launches": int(launches),
         "gpu_launches_per_step": int(kernels_per_step),
