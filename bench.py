@@ -54,6 +54,9 @@ def parse_args(argv=None):
     ap.add_argument("--sweep", default=None,
                     help="comma-separated alphas: print one line per alpha")
     ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--fit-time-model", action="store_true",
+                    help="profile tb_decode_attn over N_kv and tb_score_evict over N_x on the 7b "
+                         "shape and print the least-squares time model (Eq. 6a/6b) with its MAPE")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target seconds of oracle work for the cpu_baseline sample")
@@ -93,7 +96,8 @@ def alg_bytes(wl, n, alpha, lens):
 def stage_rooflines(wl, n, ab, stage_ms, peaks):
     """Every stage against its roofline: algorithmic bytes over the stage time
     against the measured copy bandwidth; the window scoring also as a tensor
-    contraction (2 Hq W d flops per key and pass, two passes) against the
+    contraction (2 Hq W d flops per key and pass; pass 1 over the N keys,
+    pass 2 over the P = N - W prefix keys) against the
     measured sustained bf16 rate (its kernel runs inside a long step)."""
     hbm = float(peaks["hbm_gbs"])
     out = {}
@@ -102,7 +106,7 @@ def stage_rooflines(wl, n, ab, stage_ms, peaks):
         out[s] = {"bound": "hbm", "alg_bytes": int(ab[s]), "us": round(1e3 * ms, 2),
                   "achieved_gbs": round(gbs, 1), "frac": round(gbs / hbm, 4)}
     if "window_scores" in stage_ms and wl.dtype == "bf16":
-        flops = 2 * (2.0 * wl.hq * wl.window * wl.head_dim * float(np.sum(n)))
+        flops = 2.0 * wl.hq * wl.window * wl.head_dim * float(2 * np.sum(n) - len(n) * wl.window)
         tf = flops / (stage_ms["window_scores"] * 1e-3) / 1e12
         peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
         out["window_scores"]["tensor"] = {"flops": flops, "achieved_tflops": round(tf, 1),
@@ -348,22 +352,14 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     if dist:
         dist.barrier()
     total_ms = t0.elapsed_time(t1)
-    # the same steps once more, stage by stage, with events between stages
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
-    with torch.cuda.stream(stream):
-        for i in range(K):
-            evs[i][0].record(stream)
-            for j in range(4):
-                stage_graphs[i % L][j].replay()
-                evs[i][j + 1].record(stream)
-    torch.cuda.synchronize(dev)
+    stage_ms, stage_timing = time_stages(torch, dev, stream, cap, layers, stages, stage_call,
+                                         stage_graphs, K)
     clocks = sampler.stop()
     launches = kernels_per_step * K
     total_ms = max_over_ranks(dist, total_ms, dev)
     for d in layers:
         st, raw = tb.tb_read_status(d["dws"], stream=stream)
         assert st == tb.TB_OK, raw
-    stage_ms = {s: sum(ev[j].elapsed_time(ev[j + 1]) for ev in evs) / K for j, s in enumerate(stages)}
     ms_step = total_ms / K
     value = job_value(world, ab["step"], K, total_ms)
 
@@ -377,6 +373,17 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
             "traffic": profiled_traffic(dom, wl.name),
             "alg_bytes_per_launch": ab[dom], "avg_launch_ms": round(stage_ms[dom], 5)}
+    sroof = stage_rooflines(wl, n, ab, stage_ms, peaks)
+    if "tensor" in sroof.get(dom, {}):
+        # the window scoring is a dense bf16 contraction (two QK^T passes over
+        # the window rows: statistics, then normalised sums), so its roofline
+        # is the tensor rate; its HBM fraction stays in the stage table
+        t = sroof[dom]["tensor"]
+        roof.update({"bound": "tensor", "achieved": t["achieved_tflops"], "peak": t["peak_tflops"],
+                     "unit": "TFLOP/s", "frac": t["frac"],
+                     "peak_source": "measured sustained bf16 (MEASURED_PEAKS.json bf16_tflops_sustained)",
+                     "alg_flops_per_launch": t["flops"],
+                     "flops_rule": "2 Hq W d flops per key and pass: N keys (statistics) + N - W keys (sums)", "hbm_frac": sroof[dom]["frac"]})
 
     e2e = run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R)
 
@@ -390,7 +397,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             "workload": describe(wl, n, a), "alpha": float(a[0]) if len(set(a.tolist())) == 1 else a.tolist(),
             "layers_rotated": L, "l2": "inputs larger than L2: %d rotating layer buffers of %.0f MB" % (L, layer_bytes / 1e6),
             "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
-            "launch": "each step is one CUDA-graph replay of the four C-ABI calls; stage times from per-stage graph replays with events between them",
+            "launch": "each step is one CUDA-graph replay of the four C-ABI calls",
+            "stage_timing": stage_timing,
             "parallelism": "replicas" if world > 1 else "single GPU"},
         "us_per_layer": {"evict": round(evict_us, 2), "decode": round(1e3 * stage_ms["decode_attn"], 2),
                          "step": round(1e3 * ms_step, 2),
@@ -399,13 +407,58 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                 "decode": round(ab["decode_attn"] / (stage_ms["decode_attn"] * 1e-3) / 1e9, 1)},
         "frac_of_8tbs": round(value / world / NOMINAL_HBM_GBS, 4),
         "roofline": roof,
-        "stage_roofline": stage_rooflines(wl, n, ab, stage_ms, peaks),
+        "stage_roofline": sroof,
         "e2e": e2e,
         "gpu_launches": int(launches),
         "gpu_launches_per_step": int(kernels_per_step),
         "clocks": clocks,
     }
     return res
+
+
+def time_stages(torch, dev, stream, cap, layers, stages, stage_call, stage_graphs, K):
+    """Per-stage device time. Preferred: the step graph with timing events
+    recorded as graph nodes between its kernels (each replay then times the
+    stages back to back, as the step runs them). Where the installed torch
+    cannot put timing events into a graph, the fallback replays one graph
+    per stage with events between the replays, which adds the gap between
+    graph launches to every stage."""
+    L = len(layers)
+    try:
+        timed = []
+        for d in layers:
+            evs = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(stages) + 1)]
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=cap):
+                evs[0].record(cap)
+                for j, name in enumerate(stages):
+                    stage_call(name, d, cap)
+                    evs[j + 1].record(cap)
+            timed.append((g, evs))
+        torch.cuda.synchronize(dev)
+        acc = [0.0] * len(stages)
+        with torch.cuda.stream(stream):
+            for i in range(L + K):
+                g, evs = timed[i % L]
+                g.replay()
+                torch.cuda.synchronize(dev)
+                if i >= L:   # one warm replay of every timed graph first
+                    for j in range(len(stages)):
+                        acc[j] += evs[j].elapsed_time(evs[j + 1])
+        return ({s: acc[j] / K for j, s in enumerate(stages)},
+                "timing events as nodes of the step graph, between its kernels")
+    except (TypeError, RuntimeError):
+        torch.cuda.synchronize(dev)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(K)]
+    with torch.cuda.stream(stream):
+        for i in range(K):
+            evs[i][0].record(stream)
+            for j in range(len(stages)):
+                stage_graphs[i % L][j].replay()
+                evs[i][j + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    return ({s: sum(ev[j].elapsed_time(ev[j + 1]) for ev in evs) / K for j, s in enumerate(stages)},
+            "per-stage graph replays with events between them (adds the graph launch gap)")
 
 
 def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R):
@@ -558,6 +611,135 @@ def run_reference(args, wl, alpha):
     }
 
 
+# ---------------------------------------------------------------------------
+# profiling-based fit of the time model (Eq. 6a / 6b) on these kernels
+# ---------------------------------------------------------------------------
+
+def _time_per_call(torch, dev, stream, calls, reps):
+    """Device µs per call of `calls` (a list of zero-argument launches on
+    `stream`), captured into one CUDA graph and replayed `reps` times."""
+    cap = torch.cuda.Stream(dev)
+    for c in calls:
+        c(stream)
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cap):
+        for c in calls:
+            c(cap)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.replay()
+    torch.cuda.synchronize(dev)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        t1.record(stream)
+    torch.cuda.synchronize(dev)
+    return 1e3 * t0.elapsed_time(t1) / (reps * len(calls))
+
+
+def _fit_report(tb, x, t_us, degree):
+    coef, mape = tb.tb_fit_time_model(x, t_us, degree)
+    # hold-out: fit on the even-indexed points, score the odd-indexed ones
+    ce, _ = tb.tb_fit_time_model(x[0::2], t_us[0::2], degree)
+    xo, to = np.asarray(x[1::2], np.float64), np.asarray(t_us[1::2], np.float64)
+    hold = 100.0 * float(np.mean(np.abs(np.polyval(ce, xo) - to) / to))
+    names = ["p_us_per_token", "q_us"] if degree == 1 else ["a_us_per_token2", "b_us_per_token", "c_us"]
+    rep = {k: float("%.6g" % v) for k, v in zip(names, coef)}
+    rep.update({"mape_pct": round(mape, 3), "holdout_mape_pct": round(hold, 3),
+                "points": [[int(a), round(b, 3)] for a, b in zip(x, t_us)]})
+    return rep
+
+
+def run_time_fit(args):
+    """Section "Profiling-based Fitting": measure the path's kernels over a
+    range of lengths on the paper's model shape (28 query / 4 KV heads,
+    d 128, bf16) and fit Eq. 6b to the decode attention (N_kv in 1K..32K,
+    the paper's profiling range) and Eq. 6a's quadratic to the eviction
+    (N_x in 2K..32K, alpha 0.5). Every point rotates over enough layer
+    buffers that a graph replay reads more than L2 holds."""
+    import torch
+    from paper_2512_21859_gb300 import binding as tb
+
+    tb.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    wl = inputs.WORKLOADS["7b"]
+    d, e = wl.head_dim, 2
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(wl.seed * 1000 + 6)
+    sampler = ClockSampler(0)
+
+    dec_x, dec_t = [], []
+    for n in range(1024, 32768 + 1, 1024):
+        per = 2 * wl.hkv * n * d * e
+        L = int(min(256, max(2, math.ceil(3 * L2_BYTES / per))))
+        ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=d, dtype=tb.TB_BF16, cache_offset=[0],
+                              cache_cap=[n], cache_rows=n, max_len=n)
+        dws = tb.tb_decode_workspace_size(ddesc)
+        kv = torch.randn((L, 2, wl.hkv, n, d), generator=gen, device=dev, dtype=torch.bfloat16)
+        q = torch.randn((L, 1, wl.hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+        lens = torch.full((1,), n, dtype=torch.int32, device=dev)
+        out = torch.empty((L, 1, wl.hq, d), dtype=torch.float32, device=dev)
+        ws = torch.empty((L, max(dws, 1)), dtype=torch.uint8, device=dev)
+        calls = [lambda st, l=l: tb.tb_decode_attn(ddesc, q[l], kv[l, 0], kv[l, 1], lens, out[l], ws[l],
+                                                   stream=st) for l in range(L)]
+        dec_x.append(n)
+        dec_t.append(_time_per_call(torch, dev, stream, calls, max(3, 2000 // L)))
+        for l in range(L):
+            st, raw = tb.tb_read_status(ws[l], stream=stream)
+            assert st == tb.TB_OK, raw
+        del kv, q, out, ws
+
+    ev_x, ev_t = [], []
+    alpha = 0.5
+    for n in range(2048, 32768 + 1, 2048):
+        lay = inputs.make_layer(wl, 0, alpha=alpha, n_override=[n])
+        per = 2 * wl.hkv * n * d * e
+        L = int(min(64, max(2, math.ceil(3 * L2_BYTES / per))))
+        desc = tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=d, window=wl.window, pool_k=wl.pool_k,
+                            dtype=tb.TB_BF16, n=lay["n"], alpha=lay["alpha"], kv_offset=lay["kv_offset"],
+                            kv_rows=n, out_cap=[retained(n, wl.window, alpha)[1]])
+        _, idx_rows = tb.tb_evict_layout(desc)
+        ews = tb.tb_evict_workspace_size(desc)
+
+        def dev_bf16(x):
+            return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
+
+        base = {k: dev_bf16(lay[k]) for k in ("q_win", "K", "V")}
+        bufs = []
+        for l in range(L):
+            b = {k: (v if l == 0 else v.clone()) for k, v in base.items()}
+            b["Kc"] = torch.empty((wl.hkv, desc.out_rows, d), dtype=torch.bfloat16, device=dev)
+            b["Vc"] = torch.empty_like(b["Kc"])
+            b["idx"] = torch.empty((wl.hkv, idx_rows), dtype=torch.int32, device=dev)
+            b["ws"] = torch.empty(ews, dtype=torch.uint8, device=dev)
+            bufs.append(b)
+        calls = [lambda st, b=b: tb.tb_score_evict(desc, b["q_win"], b["K"], b["V"], b["idx"], b["Kc"],
+                                                   b["Vc"], None, b["ws"], stream=st) for b in bufs]
+        ev_x.append(n)
+        ev_t.append(_time_per_call(torch, dev, stream, calls, max(3, 400 // L)))
+        for b in bufs:
+            st, raw = tb.tb_read_status(b["ws"], stream=stream)
+            assert st == tb.TB_OK, raw
+        del bufs, base
+    clocks = sampler.stop()
+    return {
+        "metric": "time-model fit (Eq. 6a / 6b by least squares) of the path's kernels, MAPE %",
+        "unit": "us", "data": "synthetic (seeded Gaussian; eviction inputs with planted heavy hitters)",
+        "config": {"workload": "7b shape: 28q/4kv heads, d=128, bf16, batch 1, W=32, pool 7",
+                   "timing": "CUDA graph of one call per rotated layer buffer (inputs larger than L2), "
+                             "CUDA events around the replays"},
+        "decode_attn_eq6b": _fit_report(tb, dec_x, dec_t, 1),
+        "score_evict_eq6a": dict(_fit_report(tb, ev_x, ev_t, 2), alpha=alpha),
+        "clocks": clocks,
+    }
+
+
 def main(argv=None):
     args = parse_args(argv)
     world, rank, local = dist_env()
@@ -572,6 +754,10 @@ def main(argv=None):
     if not torch.cuda.is_available():
         print(json.dumps({"error": "no CUDA device: the benchmark times the GPU path only"}))
         return 1
+    if args.fit_time_model:
+        if rank == 0:
+            print(json.dumps(run_time_fit(args)), flush=True)
+        return 0
     dist = dist_init(world, True)
     alphas = [float(x) for x in args.sweep.split(",")] if args.sweep else [args.alpha]
     base_cpu = None

@@ -293,6 +293,27 @@ tb_status tb_alpha_star(const tb_time_model *model, int64_t n_x, double n_hat,
                         double budget, double alpha_max, double *alpha_out,
                         int64_t *n_w_out);
 
+/*
+ * Profiling-based fitting (Section "Profiling-based Fitting" of the
+ * workload-guided execution time estimator): the least-squares polynomial
+ * through measured (x_i, t_i) pairs, in the form of Eq. 6a (degree 2:
+ * t = a x^2 + b x + c, x = N_x) or Eq. 6b (degree 1: t = p x + q,
+ * x = N_kv). Host memory, host only; no device work.
+ *  - x, t: count values each (any order, any units; t > 0).
+ *  - coef_out: degree + 1 coefficients, highest power first ({a, b, c} or
+ *    {p, q}), minimising sum_i (poly(x_i) - t_i)^2. Solved by Householder
+ *    QR on the Vandermonde columns of x / max|x| (fp64), not by the normal
+ *    equations, so N_x^2 ~ 1e9 costs no accuracy.
+ *  - mape_out (may be NULL): the fit's mean absolute percentage error over
+ *    the same points, 100 / count * sum_i |poly(x_i) - t_i| / t_i.
+ * Errors: TB_ERR_INVALID_ARG for a NULL x, t or coef_out, degree other than
+ * 1 or 2, fewer than degree + 1 distinct x values, a non-finite x or t, or
+ * some t <= 0.
+ */
+tb_status tb_fit_time_model(const double *x, const double *t, int64_t count,
+                            int32_t degree, double *coef_out,
+                            double *mape_out);
+
 #ifdef __cplusplus
 }
 #endif

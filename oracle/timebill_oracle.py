@@ -30,6 +30,10 @@ from the exact input values):
    Inference Mechanism"): the smallest alpha in [0, alpha_max] whose
    worst-case execution time estimate (Eq. 12, built from Eqs. 6a, 9-11)
    fits the budget, found here from its definition by bisection.
+9. Profiling-based fitting (Section "Profiling-based Fitting"): the
+   least-squares coefficients of Eq. 6a (degree 2) or Eq. 6b (degree 1)
+   through measured (length, time) pairs, and the fit's mean absolute
+   percentage error (the accuracy measure of the time-model evaluation).
 
 Parity status: every function here is pinned by tests/test_oracle_pins.py
 (hand-derived closed forms, brute force, invariants, library routines).
@@ -53,6 +57,7 @@ __all__ = [
     "pessimistic_length",
     "wcet",
     "alpha_star",
+    "fit_time_model",
 ]
 
 
@@ -255,3 +260,22 @@ def alpha_star(a: float, b: float, c: float, p: float, q: float, n_x: int, n_hat
         else:
             lo = mid
     return hi
+
+
+# ---------------------------------------------------------------------------
+# step 9: profiling-based fitting of the time model
+# ---------------------------------------------------------------------------
+
+def fit_time_model(x: Sequence[float], t: Sequence[float], degree: int) -> Tuple[List[float], float]:
+    """Least squares (the fitting method the paper names) of t ~ poly(x) with
+    the form of Eq. 6a (degree 2: a x^2 + b x + c) or Eq. 6b (degree 1:
+    p x + q). Returns the coefficients, highest power first, and the MAPE in
+    percent over the same points: 100/n sum |poly(x_i) - t_i| / t_i.
+    The least-squares solve is numpy's lstsq on the Vandermonde matrix."""
+    xa = np.asarray(x, dtype=np.float64)
+    ta = np.asarray(t, dtype=np.float64)
+    V = np.stack([xa ** k for k in range(degree, -1, -1)], axis=1)
+    coef = np.linalg.lstsq(V, ta, rcond=None)[0]
+    fit = V @ coef
+    mape = 100.0 * float(np.mean(np.abs(fit - ta) / ta))
+    return [float(c) for c in coef], mape

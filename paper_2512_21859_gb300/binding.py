@@ -24,7 +24,7 @@ __all__ = [
     "tb_window_scores", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
     "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_exp2",
-    "TimeModel", "tb_wcet", "tb_alpha_star",
+    "TimeModel", "tb_wcet", "tb_alpha_star", "tb_fit_time_model",
 ]
 
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
@@ -108,6 +108,7 @@ def load():
         "tb_alpha_star": (I, [P, ctypes.c_int64, ctypes.c_double, ctypes.c_double, ctypes.c_int64,
                               ctypes.c_double, ctypes.c_double, ctypes.c_double,
                               ctypes.POINTER(ctypes.c_double), _I64P]),
+        "tb_fit_time_model": (I, [_F64P, _F64P, ctypes.c_int64, ctypes.c_int32, _F64P, _F64P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -347,3 +348,17 @@ def tb_alpha_star(model: TimeModel, n_x: int, n_hat: float, k: float, n_max: int
                                 float(t_predict), float(budget), float(alpha_max), ctypes.byref(a),
                                 ctypes.byref(n_w)), "tb_alpha_star")
     return a.value, n_w.value
+
+
+def tb_fit_time_model(x, t, degree: int):
+    """Least-squares coefficients (highest power first) and MAPE in percent
+    of the Eq. 6a (degree 2) or Eq. 6b (degree 1) fit (host computation)."""
+    xa = np.ascontiguousarray(x, dtype=np.float64)
+    ta = np.ascontiguousarray(t, dtype=np.float64)
+    if xa.shape != ta.shape or xa.ndim != 1:
+        raise ValueError("x and t must be 1-D and of one length")
+    coef = (ctypes.c_double * (max(int(degree), 0) + 1))()
+    mape = ctypes.c_double()
+    _check(load().tb_fit_time_model(xa.ctypes.data_as(_F64P), ta.ctypes.data_as(_F64P), xa.size,
+                                    int(degree), coef, ctypes.byref(mape)), "tb_fit_time_model")
+    return list(coef), mape.value

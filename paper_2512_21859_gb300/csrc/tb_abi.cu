@@ -9,6 +9,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <vector>
 #include <atomic>
 
 #include "tb_internal.cuh"
@@ -330,6 +331,80 @@ tb_status tb_alpha_star(const tb_time_model* model, int64_t n_x, double n_hat, d
   }
   *alpha_out = alpha;
   if (n_w_out) *n_w_out = n_w;
+  return TB_OK;
+}
+
+// Least squares of the profiling-based fit (Eq. 6a / 6b coefficients):
+// Householder QR of the (count x (degree + 1)) Vandermonde matrix of the
+// scaled abscissae u = x / s, then back substitution; the coefficient of u^k
+// is divided by s^k at the end.
+tb_status tb_fit_time_model(const double* x, const double* t, int64_t count, int32_t degree,
+                            double* coef_out, double* mape_out) {
+  if (!x || !t || !coef_out || (degree != 1 && degree != 2) || count < degree + 1)
+    return TB_ERR_INVALID_ARG;
+  double s = 0.0;
+  for (int64_t i = 0; i < count; ++i) {
+    if (!std::isfinite(x[i]) || !std::isfinite(t[i]) || !(t[i] > 0.0)) return TB_ERR_INVALID_ARG;
+    s = std::fmax(s, std::fabs(x[i]));
+  }
+  {
+    std::vector<double> xs(x, x + count);
+    std::sort(xs.begin(), xs.end());
+    if (std::unique(xs.begin(), xs.end()) - xs.begin() < degree + 1) return TB_ERR_INVALID_ARG;
+  }
+  if (s == 0.0) s = 1.0;
+  const int nc = degree + 1;  // columns: u^degree, ..., u, 1
+  const size_t n = (size_t)count;
+  std::vector<double> A(n * nc), y(t, t + count);
+  for (size_t i = 0; i < n; ++i) {
+    const double u = x[i] / s;
+    double pw = 1.0;
+    for (int c = nc - 1; c >= 0; --c) {
+      A[i * nc + c] = pw;
+      pw *= u;
+    }
+  }
+  std::vector<double> v(n);
+  for (int c = 0; c < nc; ++c) {
+    double norm = 0.0;
+    for (size_t i = c; i < n; ++i) norm = std::hypot(norm, A[i * nc + c]);
+    if (norm == 0.0) return TB_ERR_INVALID_ARG;
+    const double alpha = A[c * nc + c] > 0.0 ? -norm : norm;
+    double vn = 0.0;
+    for (size_t i = c; i < n; ++i) {
+      v[i] = A[i * nc + c] - (i == (size_t)c ? alpha : 0.0);
+      vn += v[i] * v[i];
+    }
+    if (vn > 0.0) {
+      for (int j = c; j < nc; ++j) {
+        double d = 0.0;
+        for (size_t i = c; i < n; ++i) d += v[i] * A[i * nc + j];
+        d = 2.0 * d / vn;
+        for (size_t i = c; i < n; ++i) A[i * nc + j] -= d * v[i];
+      }
+      double d = 0.0;
+      for (size_t i = c; i < n; ++i) d += v[i] * y[i];
+      d = 2.0 * d / vn;
+      for (size_t i = c; i < n; ++i) y[i] -= d * v[i];
+    }
+  }
+  double cu[3] = {0.0, 0.0, 0.0};
+  for (int c = nc - 1; c >= 0; --c) {
+    double r = y[c];
+    for (int j = c + 1; j < nc; ++j) r -= A[c * nc + j] * cu[j];
+    if (A[c * nc + c] == 0.0) return TB_ERR_INVALID_ARG;
+    cu[c] = r / A[c * nc + c];
+  }
+  for (int c = 0; c < nc; ++c) coef_out[c] = cu[c] / std::pow(s, (double)(nc - 1 - c));
+  if (mape_out) {
+    double acc = 0.0;
+    for (size_t i = 0; i < n; ++i) {
+      double f = 0.0;
+      for (int c = 0; c < nc; ++c) f = f * x[i] + coef_out[c];
+      acc += std::fabs(f - t[i]) / t[i];
+    }
+    *mape_out = 100.0 * acc / (double)n;
+  }
   return TB_OK;
 }
 

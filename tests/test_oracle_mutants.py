@@ -36,6 +36,9 @@ MUTANTS = {
     "per-step constant dropped": ("t_decode += p * ((1.0 - alpha) * n_x + i - 1) + q", "t_decode += p * ((1.0 - alpha) * n_x + i - 1)"),
     "pessimistic length rounded down": ("int(min(math.ceil(k * n_hat), n_max))", "int(min(math.floor(k * n_hat), n_max))"),
     "predictor overhead ignored": ("return t_predict + wcet(a, b, c, p, q, n_x, al, n_w) - budget", "return wcet(a, b, c, p, q, n_x, al, n_w) - budget"),
+    "fit without the constant column": ("for k in range(degree, -1, -1)], axis=1)", "for k in range(degree, 0, -1)], axis=1)"),
+    "MAPE relative to the fit": ("np.abs(fit - ta) / ta", "np.abs(fit - ta) / fit"),
+    "MAPE without the percent": ("mape = 100.0 * float(", "mape = float("),
 }
 
 
@@ -90,6 +93,10 @@ def _pins_pass(m):
         al = m.alpha_star(1e-9, 2e-6, 1e-4, 1e-6, 5e-5, 1000, 10, 1.0, 100, 3e-4, 8e-3, 0.95)
         want = 1.0 - (8e-3 - 3e-4 - (1e-3 + 2e-3 + 1e-4) - 9 * 5e-5 - 36e-6) / 9e-3
         if abs(al - want) > 1e-12 or m.pessimistic_length(10, 1.25, 100) != 13:
+            return False
+        # the least-squares fit: the hand line of tests/test_time_fit.py
+        coef, mape = m.fit_time_model([0, 1, 2], [1, 3, 2], 1)
+        if not np.allclose(coef, [0.5, 1.5], atol=1e-14) or abs(mape - 100.0 * (0.5 + 1 / 3 + 0.25) / 3) > 1e-12:
             return False
         return True
     except (ValueError, IndexError, AssertionError):
