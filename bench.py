@@ -417,19 +417,23 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
 
 
 def time_stages(torch, dev, stream, cap, layers, stages, stage_call, stage_graphs, K):
-    """Per-stage device time. Preferred: the step graph with timing events
-    recorded as graph nodes between its kernels (each replay then times the
-    stages back to back, as the step runs them). Where the installed torch
-    cannot put timing events into a graph, the fallback replays one graph
-    per stage with events between the replays, which adds the gap between
-    graph launches to every stage."""
+    """Per-stage device time. Preferred: timing events recorded as graph
+    nodes between the kernels of a step, in a graph that first runs the
+    previous layer's step untimed, so that the timed step starts behind
+    running work as it does when step graphs are replayed back to back (not
+    behind the start-up of a graph on an idle GPU). Where the installed
+    torch cannot put timing events into a graph, the fallback replays one
+    graph per stage with events between the replays, which adds the gap
+    between graph launches to every stage."""
     L = len(layers)
     try:
         timed = []
-        for d in layers:
+        for li, d in enumerate(layers):
             evs = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(stages) + 1)]
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, stream=cap):
+                for name in stages:
+                    stage_call(name, layers[li - 1], cap)
                 evs[0].record(cap)
                 for j, name in enumerate(stages):
                     stage_call(name, d, cap)
@@ -446,7 +450,7 @@ def time_stages(torch, dev, stream, cap, layers, stages, stage_call, stage_graph
                     for j in range(len(stages)):
                         acc[j] += evs[j].elapsed_time(evs[j + 1])
         return ({s: acc[j] / K for j, s in enumerate(stages)},
-                "timing events as nodes of the step graph, between its kernels")
+                "timing events as graph nodes between the kernels of a step that follows another step")
     except (TypeError, RuntimeError):
         torch.cuda.synchronize(dev)
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(K)]

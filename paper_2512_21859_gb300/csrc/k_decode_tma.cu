@@ -122,19 +122,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int r0 = lane >> 2, qd = lane & 3;  // fragment row (and row + 8), column pair
-  int len = lens[b];
-  {
-    const int64_t cap64 = p.max_len < (int64_t)p.cache_cap[b] ? p.max_len : (int64_t)p.cache_cap[b];
-    if (len > (int)cap64) {
-      if (split == 0 && g == 0 && tid == 0) atomicOr(status, kStatusRange);
-      len = (int)cap64;
-    }
-    if (len < 0) len = 0;
-  }
+  // The first tiles are requested before the length is read (its load
+  // would delay them by a memory round trip): they cover the split's rows up
+  // to the request's cap, which lie inside its slice of the cache; tiles
+  // past the length are waited for and dropped after the key loop.
   const int k0 = split * p.split_len;
-  const int k1 = min(len, k0 + p.split_len);
-  const int ntiles = k1 > k0 ? (k1 - k0 + kTile - 1) / kTile : 0;
-  const size_t part_base = ((size_t)b * p.hq + (size_t)g * G) * p.splits + split;
+  const int64_t cap64 = p.max_len < (int64_t)p.cache_cap[b] ? p.max_len : (int64_t)p.cache_cap[b];
+  const int k1c = (int)min((int64_t)k0 + p.split_len, cap64);
+  const int ntiles_c = k1c > k0 ? (k1c - k0 + kTile - 1) / kTile : 0;
   const int row0 = (int)((int64_t)g * p.cache_rows + p.cache_off[b]) + k0;
 
   if (tid == 0) {
@@ -158,8 +153,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     tc::tma_prefetch_desc(&tk);
     tc::tma_prefetch_desc(&tv);
-    for (; issued < kStages && issued < ntiles; ++issued) issue(issued);
+    for (; issued < kStages && issued < ntiles_c; ++issued) issue(issued);
   }
+  int len = lens[b];
+  if (len > (int)cap64) {
+    if (split == 0 && g == 0 && tid == 0) atomicOr(status, kStatusRange);
+    len = (int)cap64;
+  }
+  if (len < 0) len = 0;
+  const int k1 = min(len, k0 + p.split_len);
+  const int ntiles = k1 > k0 ? (k1 - k0 + kTile - 1) / kTile : 0;  // <= ntiles_c
+  const size_t part_base = ((size_t)b * p.hq + (size_t)g * G) * p.splits + split;
 
   // Q fragments (rows >= G are zero queries)
   uint32_t aq[KS][4];
@@ -300,6 +304,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
 
+  // tiles requested past the length (only ever among the first kStages):
+  // their copies land before the ring is reused for the merge
+  if (ok && tid == 0) {
+    for (int t = ntiles; t < issued; ++t) {
+      int dummy = 0;
+      if (!tc::mbar_wait(&full[t % kStages], (uint32_t)((t / kStages) & 1), &dummy, status)) break;
+    }
+  }
+  if (ok) __syncthreads();
   if (!ok) {
     if (tid == 0) {
       // drain the copies still in flight before the CTA exits
@@ -383,19 +396,34 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (!*last_flag) return;
   __threadfence();
   const size_t head0 = ((size_t)b * p.hq + (size_t)g * G) * p.splits;
-  // per head: weight of split s = 2^(m_s - M) / L, lanes over splits
+  // per head: weight of split s = 2^(m_s - M) / L, lanes over splits; the
+  // (m, l) pairs of the first 64 splits are loaded once and kept
   float* wts = reinterpret_cast<float*>(smem);  // [G][splits] (the ring is free)
   for (int h = warp; h < G; h += kThreads / 32) {
     const size_t hb = head0 + (size_t)h * p.splits;
+    float2 ml[2];
     float M = -INFINITY;
-    for (int sp = lane; sp < p.splits; sp += 32) M = fmaxf(M, __ldcg(&part_ml[hb + sp]).x);
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int sp = lane + 32 * i;
+      ml[i] = sp < p.splits ? __ldcg(&part_ml[hb + sp]) : make_float2(-INFINITY, 0.f);
+      M = fmaxf(M, ml[i].x);
+    }
+    for (int sp = lane + 64; sp < p.splits; sp += 32) M = fmaxf(M, __ldcg(&part_ml[hb + sp]).x);
     for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
     float L = 0.f;
-    for (int sp = lane; sp < p.splits; sp += 32) {
-      const float2 ml = __ldcg(&part_ml[hb + sp]);
-      const float wgt = (M != -INFINITY && ml.y > 0.f) ? fast_exp2(ml.x - M) : 0.f;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int sp = lane + 32 * i;
+      const float wgt = (M != -INFINITY && ml[i].y > 0.f) ? fast_exp2(ml[i].x - M) : 0.f;
+      if (sp < p.splits) wts[h * p.splits + sp] = wgt;
+      L = fmaf(ml[i].y, wgt, L);
+    }
+    for (int sp = lane + 64; sp < p.splits; sp += 32) {
+      const float2 m2 = __ldcg(&part_ml[hb + sp]);
+      const float wgt = (M != -INFINITY && m2.y > 0.f) ? fast_exp2(m2.x - M) : 0.f;
       wts[h * p.splits + sp] = wgt;
-      L = fmaf(ml.y, wgt, L);
+      L = fmaf(m2.y, wgt, L);
     }
     for (int off = 16; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
     const float inv = L > 0.f ? 1.f / L : 0.f;
@@ -403,15 +431,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int sp = lane; sp < p.splits; sp += 32) wts[h * p.splits + sp] *= inv;
   }
   __syncthreads();
-  // outputs in float4 groups of dims; every split's partial is an independent load
+  // outputs in float4 groups of dims; the splits are divided among the
+  // threads that share an output (NS of them), their sums combined by shuffles
   constexpr int D4 = D / 4;
-  for (int e = tid; e < G * D4; e += kThreads) {
+  // (G * D4 * NS is a multiple of 32 for every supported G and D, so each
+  // warp's lanes run the same iterations and the shuffles see full warps)
+  constexpr int kPer = kThreads / (G * D4);
+  constexpr int NS = kPer >= 8 ? 8 : kPer >= 4 ? 4 : kPer >= 2 ? 2 : 1;
+  static_assert((G * D4 * NS) % 32 == 0, "output groups must fill whole warps");
+  for (int e0 = tid; e0 < G * D4 * NS; e0 += kThreads) {
+    const int e = e0 / NS, part = e0 % NS;
     const int h = e / D4, d4 = e % D4;
     const size_t hb = head0 + (size_t)h * p.splits;
     const float* wh = wts + h * p.splits;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 16
-    for (int sp = 0; sp < p.splits; ++sp) {
+#pragma unroll 8
+    for (int sp = part; sp < p.splits; sp += NS) {
       const float wgt = wh[sp];
       const float4 ov = __ldcg(reinterpret_cast<const float4*>(part_o + (hb + sp) * D) + d4);
       acc.x = fmaf(ov.x, wgt, acc.x);
@@ -419,6 +454,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       acc.z = fmaf(ov.z, wgt, acc.z);
       acc.w = fmaf(ov.w, wgt, acc.w);
     }
+#pragma unroll
+    for (int off = 1; off < NS; off <<= 1) {
+      acc.x += __shfl_xor_sync(0xffffffffu, acc.x, off);
+      acc.y += __shfl_xor_sync(0xffffffffu, acc.y, off);
+      acc.z += __shfl_xor_sync(0xffffffffu, acc.z, off);
+      acc.w += __shfl_xor_sync(0xffffffffu, acc.w, off);
+    }
+    if (part != 0) continue;
     const size_t oi = ((size_t)b * p.hq + (size_t)g * G + h) * D + 4 * d4;
     if (p.out_dtype == TB_F32) {
       *reinterpret_cast<float4*>(static_cast<float*>(out) + oi) = acc;

@@ -90,6 +90,10 @@ bool make_bf16_map(CUtensorMap* map, const void* base, int d, uint64_t rows, int
 // Adds n to the process-wide launch counter (tb_launch_counter).
 void count_launches(int n);
 
+// Zeroes the first `bytes` (a multiple of 16) of a workspace on stream s
+// with one small kernel.
+cudaError_t clear_control_words(void* ws, size_t bytes, cudaStream_t s);
+
 // ---------------------------------------------------------------------------
 // launchers (each returns cudaGetLastError() of its launch)
 // ---------------------------------------------------------------------------

@@ -70,7 +70,7 @@ extern "C" tb_status tb_decode_attn_noalloc(const tb_decode_desc* desc, const vo
   char* base = static_cast<char*>(ws);
   // the split partials are fully rewritten by every call; the status word and
   // the split counters (everything before the partials) must start at zero
-  if ((st = cuda_status(cudaMemsetAsync(base, 0, w.part_o, s))) != TB_OK) return st;
+  if ((st = cuda_status(clear_control_words(base, w.part_o, s))) != TB_OK) return st;
   return cuda_status(launch_decode(p, q, Kc, Vc, lens, out,
                                    reinterpret_cast<float*>(base + w.part_o),
                                    reinterpret_cast<float2*>(base + w.part_ml),
