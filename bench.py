@@ -312,7 +312,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         st, raw = tb.tb_read_status(d["ews"], stream=stream)
         assert st == tb.TB_OK, raw
     cap = torch.cuda.Stream(dev)
-    step_graphs, stage_graphs = [], []
+    step_graphs = []
     kernels_per_step = None
     for d in layers:
         g = torch.cuda.CUDAGraph()
@@ -322,13 +322,6 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                 stage_call(name, d, cap)
         kernels_per_step = tb.tb_launch_counter() - c0
         step_graphs.append(g)
-        per = []
-        for name in stages:
-            gs = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(gs, stream=cap):
-                stage_call(name, d, cap)
-            per.append(gs)
-        stage_graphs.append(per)
     torch.cuda.synchronize(dev)
 
     with torch.cuda.stream(stream):
@@ -352,8 +345,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     if dist:
         dist.barrier()
     total_ms = t0.elapsed_time(t1)
-    stage_ms, stage_timing = time_stages(torch, dev, stream, cap, layers, stages, stage_call,
-                                         stage_graphs, K)
+    stage_ms, stage_timing = time_stages(torch, dev, stream, cap, layers, stages, stage_call, K)
     clocks = sampler.stop()
     launches = kernels_per_step * K
     total_ms = max_over_ranks(dist, total_ms, dev)
@@ -385,6 +377,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                      "alg_flops_per_launch": t["flops"],
                      "flops_rule": "2 Hq W d flops per key and pass: N keys (statistics) + N - W keys (sums)", "hbm_frac": sroof[dom]["frac"]})
 
+    lse_var = time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, ms_step, n, peaks)
+
     e2e = run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R)
 
     evict_us = 1e3 * (stage_ms["window_scores"] + stage_ms["select_topk"] + stage_ms["gather_kv"])
@@ -408,6 +402,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         "frac_of_8tbs": round(value / world / NOMINAL_HBM_GBS, 4),
         "roofline": roof,
         "stage_roofline": sroof,
+        "prefill_lse_variant": lse_var,
         "e2e": e2e,
         "gpu_launches": int(launches),
         "gpu_launches_per_step": int(kernels_per_step),
@@ -416,53 +411,111 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     return res
 
 
-def time_stages(torch, dev, stream, cap, layers, stages, stage_call, stage_graphs, K):
-    """Per-stage device time. Preferred: timing events recorded as graph
-    nodes between the kernels of a step, in a graph that first runs the
-    previous layer's step untimed, so that the timed step starts behind
-    running work as it does when step graphs are replayed back to back (not
-    behind the start-up of a graph on an idle GPU). Where the installed
-    torch cannot put timing events into a graph, the fallback replays one
-    graph per stage with events between the replays, which adds the gap
-    between graph launches to every stage."""
-    L = len(layers)
+def window_lse_torch(torch, wl, lay, dev):
+    """Input preparation for the one-pass variant (plain PyTorch, untimed):
+    each window row's natural-log sum of exp over the keys it sees, as a
+    causal prefill attention hands it over. [B][Hq][W] float32."""
+    B, G, W = len(lay["n"]), wl.group, wl.window
+    out = torch.empty((B, wl.hq, W), dtype=torch.float32, device=dev)
+
+    def f32(x):
+        if wl.dtype == "bf16":
+            return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev).float()
+        return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+    q = f32(lay["q_win"])
+    for b in range(B):
+        n, off = int(lay["n"][b]), int(lay["kv_offset"][b])
+        P = n - W
+        mask = torch.arange(n, device=dev)[None, :] > (P + torch.arange(W, device=dev))[:, None]
+        for g in range(wl.hkv):
+            Kg = f32(lay["K"][g, off:off + n])
+            s = torch.matmul(q[b, g * G:(g + 1) * G], Kg.t()) / math.sqrt(wl.head_dim)
+            s.masked_fill_(mask[None], float("-inf"))
+            out[b, g * G:(g + 1) * G] = torch.logsumexp(s, dim=-1)
+            del s, Kg
+    return out
+
+
+def time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, step_ms, n, peaks):
+    """tb_window_scores_lse (one QK^T pass, the window rows' normalisers
+    given by the prefill) timed on the same rotated layers, and the step it
+    gives with the other stages as measured."""
+    prev = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
     try:
-        timed = []
-        for li, d in enumerate(layers):
-            evs = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(stages) + 1)]
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=cap):
-                for name in stages:
-                    stage_call(name, layers[li - 1], cap)
-                evs[0].record(cap)
-                for j, name in enumerate(stages):
-                    stage_call(name, d, cap)
-                    evs[j + 1].record(cap)
-            timed.append((g, evs))
-        torch.cuda.synchronize(dev)
-        acc = [0.0] * len(stages)
-        with torch.cuda.stream(stream):
-            for i in range(L + K):
-                g, evs = timed[i % L]
-                g.replay()
-                torch.cuda.synchronize(dev)
-                if i >= L:   # one warm replay of every timed graph first
-                    for j in range(len(stages)):
-                        acc[j] += evs[j].elapsed_time(evs[j + 1])
-        return ({s: acc[j] / K for j, s in enumerate(stages)},
-                "timing events as graph nodes between the kernels of a step that follows another step")
-    except (TypeError, RuntimeError):
-        torch.cuda.synchronize(dev)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(K)]
-    with torch.cuda.stream(stream):
-        for i in range(K):
-            evs[i][0].record(stream)
-            for j in range(len(stages)):
-                stage_graphs[i % L][j].replay()
-                evs[i][j + 1].record(stream)
+        lse = window_lse_torch(torch, wl, lay, dev)
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = prev
+    cap = torch.cuda.Stream(dev)
+    for d in layers:
+        tb.tb_window_scores_lse(desc, d["q_win"], d["K"], lse, d["scores"], d["ews"], stream=stream)
     torch.cuda.synchronize(dev)
-    return ({s: sum(ev[j].elapsed_time(ev[j + 1]) for ev in evs) / K for j, s in enumerate(stages)},
-            "per-stage graph replays with events between them (adds the graph launch gap)")
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cap):
+        for d in layers:
+            tb.tb_window_scores_lse(desc, d["q_win"], d["K"], lse, d["scores"], d["ews"], stream=cap)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.replay()
+    torch.cuda.synchronize(dev)
+    reps = max(3, 60 // len(layers))
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        t1.record(stream)
+    torch.cuda.synchronize(dev)
+    for d in layers:
+        st, raw = tb.tb_read_status(d["ews"], stream=stream)
+        assert st == tb.TB_OK, raw
+    us = 1e3 * t0.elapsed_time(t1) / (reps * len(layers))
+    flops = 2.0 * wl.hq * wl.window * wl.head_dim * float(np.sum(n) - len(n) * wl.window)
+    tf = flops / (us * 1e-6) / 1e12
+    peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+    # the step with this call in place of tb_window_scores: the measured step
+    # time less the difference of the two calls' stage times
+    step = 1e3 * (step_ms - stage_ms["window_scores"]) + us
+    return {"call": "tb_window_scores_lse", "us": round(us, 2),
+            "timing": "CUDA graph of one call per rotated layer buffer, events around the replays",
+            "flops": flops, "achieved_tflops": round(tf, 1), "tensor_frac": round(tf / peak, 4),
+            "step_us_with_it": round(step, 2),
+            "note": "one QK^T pass over the prefix keys; the window rows' log-sum-exp comes from the prefill"}
+
+
+def time_stages(torch, dev, stream, cap, layers, stages, stage_call, K):
+    """Per-stage device time per launch: for each stage one CUDA graph of
+    that stage's call on every rotated layer buffer in turn (inputs larger
+    than L2 across the rotation), replayed with CUDA events around the
+    replays. This is the stage's launch duration plus the gap between two
+    kernels of a graph; the step graph's own time (the headline) also holds
+    the interaction between stages (e.g. the L2 write-back of the gather's
+    output while the next decode reads)."""
+    L = len(layers)
+    reps = max(3, -(-K // L))
+    out = {}
+    for name in stages:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap):
+            for d in layers:
+                stage_call(name, d, cap)
+        with torch.cuda.stream(stream):
+            for _ in range(2):
+                g.replay()
+        torch.cuda.synchronize(dev)
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            t1.record(stream)
+        torch.cuda.synchronize(dev)
+        out[name] = t0.elapsed_time(t1) / (reps * L)
+    return out, ("per stage: one CUDA graph of the stage's call on each of the %d rotated layer "
+                 "buffers, %d replays between CUDA events" % (L, reps))
 
 
 def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R):

@@ -138,6 +138,26 @@ tb_status tb_window_scores(const tb_evict_desc *desc, const void *q_win,
                            size_t workspace_bytes, tb_stream_t stream);
 
 /*
+ * tb_window_scores for a caller whose prefill attention already produced the
+ * log-sum-exp of the observation-window rows (eviction runs right after the
+ * prefill, Section "End-to-end Execution Time Prediction"; a flash-style
+ * prefill kernel returns this per query row). With the row statistics
+ * given, the scores need one Q K^T pass over the prefix keys instead of two:
+ *   scores[g][j] = sum_{h in g, w < W} exp(q_win[h][w] . K[g][j] / sqrt(d)
+ *                                          - lse[b][h][w]).
+ * lse: device f32 [batch][Hq][W], 4-byte aligned: the natural log of
+ * sum_{j' <= P_b + w} exp(q_win[h][w] . K[g][j'] / sqrt(d)) (the causal
+ * window rows of tb_window_scores; with these values both calls give the
+ * same scores up to rounding). Non-finite lse values give non-finite
+ * scores; nothing checks them. Other arguments, outputs and errors as in
+ * tb_window_scores; the workspace is the one tb_evict_workspace_size gives.
+ */
+tb_status tb_window_scores_lse(const tb_evict_desc *desc, const void *q_win,
+                               const void *K, const float *lse, float *scores,
+                               void *workspace, size_t workspace_bytes,
+                               tb_stream_t stream);
+
+/*
  * Steps 4-5: max-pool of the scores (kernel pool_k, stride 1, out-of-range
  * neighbours ignored), then per request and KV head the k_b prefix positions
  * with the largest pooled score (ties to the lower index) followed by the

@@ -18,7 +18,9 @@ from the exact input values):
 3. Row softmax over the visible keys, then the score of prefix key j is the
    sum of its probabilities over the window rows and the group's query heads
    (SnapKV-style observation-window voting; the paper names SnapKV as its
-   eviction method in "Experimental Setup").
+   eviction method in "Experimental Setup"). The same sums from given row
+   log-sum-exp values (a prefill attention's normalisers) are
+   window_scores_from_lse; window_lse computes those normalisers.
 4. 1-D max-pool of the scores with an odd kernel, stride 1, same padding
    (out-of-range neighbours ignored).
 5. The k prefix positions with the largest pooled score, ties to the lower
@@ -48,6 +50,8 @@ import numpy as np
 __all__ = [
     "retained_count",
     "window_scores",
+    "window_lse",
+    "window_scores_from_lse",
     "max_pool",
     "select_indices",
     "gather_rows",
@@ -107,6 +111,48 @@ def window_scores(q_win: np.ndarray, K: np.ndarray) -> np.ndarray:
             e = np.exp(logits - m)
             prob = e / e.sum(axis=1, keepdims=True)
             S[g] += prob[:, :P].sum(axis=0)
+    return S
+
+
+def window_lse(q_win: np.ndarray, K: np.ndarray) -> np.ndarray:
+    """Log-sum-exp of every window row's logits over the keys it sees: the
+    softmax normaliser of the attention definition, log sum_j exp(s_j), for
+    row w of head h over keys j <= P + w (what a causal prefill attention
+    produces for the last W query rows). Returns [Hq][W] (fp64)."""
+    q = np.asarray(q_win, dtype=np.float64)
+    k = np.asarray(K, dtype=np.float64)
+    hq, W, d = q.shape
+    hkv, N, _ = k.shape
+    G = hq // hkv
+    P = N - W
+    sigma = 1.0 / math.sqrt(d)
+    # row w's last visible key is its own position P + w
+    last_seen = P + np.arange(W)
+    visible = np.arange(N)[None, :] <= last_seen[:, None]
+    out = np.zeros((hq, W), dtype=np.float64)
+    for h in range(hq):
+        logits = np.where(visible, sigma * (q[h] @ k[h // G].T), -np.inf)
+        m = logits.max(axis=1)
+        out[h] = m + np.log(np.exp(logits - m[:, None]).sum(axis=1))
+    return out
+
+
+def window_scores_from_lse(q_win: np.ndarray, K: np.ndarray, lse: np.ndarray) -> np.ndarray:
+    """Step 3 with the row normalisers given: S[g, j] = sum over the heads h
+    of group g and window rows w of exp(s_hwj - lse[h, w]), prefix keys
+    j < P (all of them visible to every window row). Returns [Hkv][P]."""
+    q = np.asarray(q_win, dtype=np.float64)
+    k = np.asarray(K, dtype=np.float64)
+    L = np.asarray(lse, dtype=np.float64)
+    hq, W, d = q.shape
+    hkv, N, _ = k.shape
+    G = hq // hkv
+    P = N - W
+    sigma = 1.0 / math.sqrt(d)
+    S = np.zeros((hkv, P), dtype=np.float64)
+    for h in range(hq):
+        logits = sigma * (q[h] @ k[h // G, :P].T)      # [W][P]
+        S[h // G] += np.exp(logits - L[h][:, None]).sum(axis=0)
     return S
 
 

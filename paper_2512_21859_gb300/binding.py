@@ -21,7 +21,7 @@ __all__ = [
     "TbError", "EvictDesc", "DecodeDesc", "library_path", "load",
     "tb_status_string", "tb_abi_version", "tb_last_error_detail", "tb_launch_counter",
     "tb_retained_count", "tb_evict_layout", "tb_evict_workspace_size",
-    "tb_window_scores", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
+    "tb_window_scores", "tb_window_scores_lse", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
     "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_exp2",
     "TimeModel", "tb_wcet", "tb_alpha_star", "tb_fit_time_model",
@@ -96,6 +96,7 @@ def load():
         "tb_evict_layout": (I, [P, _I64P, _I64P]),
         "tb_evict_workspace_size": (I, [P, ctypes.POINTER(SZ)]),
         "tb_window_scores": (I, [P, P, P, P, P, SZ, P]),
+        "tb_window_scores_lse": (I, [P, P, P, P, P, P, SZ, P]),
         "tb_select_topk": (I, [P, P, P, P, P, SZ, P]),
         "tb_gather_kv": (I, [P, P, P, P, P, P, P]),
         "tb_score_evict": (I, [P, P, P, P, P, P, P, P, P, SZ, P]),
@@ -277,6 +278,14 @@ def tb_window_scores(desc: EvictDesc, q_win, K, scores, workspace, workspace_byt
     w, wb = _ws(workspace, workspace_bytes)
     _check(load().tb_window_scores(desc.ref(), _ptr(q_win), _ptr(K), _ptr(scores), w, wb,
                                    _stream(stream)), "tb_window_scores")
+
+
+def tb_window_scores_lse(desc: EvictDesc, q_win, K, lse, scores, workspace, workspace_bytes=None,
+                         stream=None):
+    """Window scores from the caller's window-row log-sum-exp (one QK^T pass)."""
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_window_scores_lse(desc.ref(), _ptr(q_win), _ptr(K), _ptr(lse), _ptr(scores), w,
+                                       wb, _stream(stream)), "tb_window_scores_lse")
 
 
 def tb_select_topk(desc: EvictDesc, scores, idx, pooled, workspace, workspace_bytes=None, stream=None):

@@ -15,6 +15,8 @@
 #include <cuda_runtime.h>
 #include <math.h>
 
+#include <type_traits>
+
 #include "tb_internal.cuh"
 
 namespace tb {
@@ -169,7 +171,7 @@ __global__ void __launch_bounds__(256) ws_scores_simt(const __grid_constant__ Ev
     __syncthreads();
     stage_rows<T, D>(Qs, Qg + (size_t)rb * D, M - rb, kRowsPerBlock);
     for (int e = threadIdx.x; e < kRowsPerBlock; e += blockDim.x)
-      Cs[e] = rb + e < M ? Cg[rb + e] : 0.f;
+      Cs[e] = rb + e < M ? Cg[rb + e] * p.rowc_scale : 0.f;
     for (int jt = j0; jt < j1; jt += kKeysPerTile) {
       __syncthreads();
       stage_rows<T, D>(Ks, Kg + (size_t)jt * D, j1 - jt, kKeysPerTile);
@@ -215,6 +217,22 @@ cudaError_t launch_window_combine(const EvictParams& p, const float2* partial, f
   ws_combine<<<p.batch * p.hkv, 256, 0, s>>>(p, partial, rowc);
   count_launches(1);
   return cudaGetLastError();
+}
+
+cudaError_t launch_window_votes_simt(const EvictParams& p, const void* q_win, const void* K,
+                                     float* scores, const float* rowc, cudaStream_t s) {
+  auto go = [&](auto kern, auto qt) {
+    using T = std::remove_const_t<std::remove_pointer_t<decltype(qt)>>;
+    kern<<<p.items, 256, 0, s>>>(p, static_cast<const T*>(q_win), static_cast<const T*>(K), rowc,
+                                 scores);
+    count_launches(1);
+    return cudaGetLastError();
+  };
+  if (p.dtype == TB_F32)
+    return p.d == 64 ? go(ws_scores_simt<float, 64>, (const float*)nullptr)
+                     : go(ws_scores_simt<float, 128>, (const float*)nullptr);
+  return p.d == 64 ? go(ws_scores_simt<uint16_t, 64>, (const uint16_t*)nullptr)
+                   : go(ws_scores_simt<uint16_t, 128>, (const uint16_t*)nullptr);
 }
 
 cudaError_t launch_window_scores_simt(const EvictParams& p, const void* q_win, const void* K,

@@ -250,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (MODE == kPassVotes)
     for (int r = threadIdx.x; r < 256; r += blockDim.x)
-      ncr[r] = r < M ? -rowc[segrow + r] : -INFINITY;
+      ncr[r] = r < M ? -(rowc[segrow + r] * p.rowc_scale) : -INFINITY;
 
   // ---- set-up: barriers and the TMEM allocation
   if (threadIdx.x == 0) {
@@ -754,6 +754,28 @@ cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, con
     return cudaErrorInvalidValue;
   return p.d == 64 ? launch_tc_typed<64>(pt, tq, tk, scores, partial, rowc, status, tilectr, s)
                    : launch_tc_typed<128>(pt, tq, tk, scores, partial, rowc, status, tilectr, s);
+}
+
+cudaError_t launch_window_votes_tc(const EvictParams& p, const void* q_win, const void* K,
+                                   float* scores, const float* rowc, int32_t* status,
+                                   int32_t* tilectr, cudaStream_t s) {
+  const EvictParams pt = tc_item_params(p);
+  CUtensorMap tq, tk;
+  const uint64_t qrows = (uint64_t)p.batch * p.hq * p.window;
+  const uint64_t krows = (uint64_t)p.hkv * p.kv_rows;
+  if (!make_bf16_map(&tq, q_win, p.d, qrows, 128) || !make_bf16_map(&tk, K, p.d, krows, 128))
+    return cudaErrorInvalidValue;
+  uint32_t* gsync = reinterpret_cast<uint32_t*>(status) + kGridSyncWord;
+  auto launch = [&](auto kern, int smem) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    kern<<<pt.items, kThreads, smem, s>>>(pt, tq, tk, nullptr, rowc, scores, status, gsync,
+                                           tilectr);
+    count_launches(1);
+    return cudaGetLastError();
+  };
+  return p.d == 64 ? launch(ws_tc<64, kPassVotes>, Geo<64>::kSmem)
+                   : launch(ws_tc<128, kPassVotes>, Geo<128>::kSmem);
 }
 
 }  // namespace tb

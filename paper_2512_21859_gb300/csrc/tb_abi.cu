@@ -85,6 +85,7 @@ tb_status build_evict(const tb_evict_desc* d, EvictParams* p) {
   p->kv_rows = d->kv_rows;
   p->out_rows = d->out_rows;
   p->scale_log2 = (float)(1.4426950408889634 / sqrt((double)d->head_dim));
+  p->rowc_scale = 1.0f;
 
   int64_t score_rows = 0, idx_rows = 0, items = 0;
   int64_t rlen[TB_MAX_BATCH];
@@ -260,6 +261,14 @@ cudaError_t clear_control_words(void* ws, size_t bytes, cudaStream_t s) {
   clear_words<<<blocks, 256, 0, s>>>(static_cast<uint4*>(ws), n16);
   count_launches(1);
   return cudaGetLastError();
+}
+
+cudaError_t launch_window_votes(const EvictParams& p, const void* q_win, const void* K,
+                                float* scores, const float* rowc, int32_t* status,
+                                int32_t* tilectr, cudaStream_t s) {
+  if (window_scores_tc_supported(p))
+    return launch_window_votes_tc(p, q_win, K, scores, rowc, status, tilectr, s);
+  return launch_window_votes_simt(p, q_win, K, scores, rowc, s);
 }
 
 cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
@@ -461,6 +470,24 @@ tb_status tb_window_scores(const tb_evict_desc* desc, const void* q_win, const v
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if ((st = cuda_status(clear_control_words(workspace, w.zeroed, s))) != TB_OK) return st;
   return run_window_scores(p, w, q_win, K, scores, workspace, s);
+}
+
+tb_status tb_window_scores_lse(const tb_evict_desc* desc, const void* q_win, const void* K,
+                               const float* lse, float* scores, void* workspace,
+                               size_t workspace_bytes, tb_stream_t stream) {
+  EvictParams p;
+  tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  if (!q_win || !K || !lse || !scores || !aligned16(q_win) || !aligned16(K) ||
+      !aligned16(scores) || (reinterpret_cast<uintptr_t>(lse) & 3u) != 0)
+    return TB_ERR_INVALID_ARG;
+  const EvictWorkspace w = carve_evict(p);
+  if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = cuda_status(clear_control_words(workspace, w.zeroed, s))) != TB_OK) return st;
+  p.rowc_scale = 1.4426950408889634f;  // natural-log LSE -> log2 units
+  return cuda_status(launch_window_votes(p, q_win, K, scores, lse, at<int32_t>(workspace, w.status),
+                                         at<int32_t>(workspace, w.tilectr), s));
 }
 
 tb_status tb_select_topk(const tb_evict_desc* desc, const float* scores, int32_t* idx,

@@ -48,7 +48,9 @@ struct EvictParams {
   int32_t pad0;
   int64_t kv_rows, out_rows, score_rows, idx_rows;
   float scale_log2;   // log2(e) / sqrt(d)
-  int32_t pad1;
+  float rowc_scale;   // c_row = rowc[r] * rowc_scale in log2 units: 1 for the
+                      // library's own statistics, log2(e) for a caller's
+                      // natural-log LSE (tb_window_scores_lse)
   EvictReq req[TB_MAX_BATCH];
 };
 
@@ -100,6 +102,11 @@ cudaError_t clear_control_words(void* ws, size_t bytes, cudaStream_t s);
 cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
                                  float* scores, float2* partial, float* rowc,
                                  int32_t* status, int32_t* tilectr, cudaStream_t s);
+// The normalised window sums alone, from given per-row log2-sum-exp values
+// (rowc [B][Hkv][G*W], scaled by p.rowc_scale): one QK^T pass.
+cudaError_t launch_window_votes(const EvictParams& p, const void* q_win, const void* K,
+                                float* scores, const float* rowc, int32_t* status,
+                                int32_t* tilectr, cudaStream_t s);
 cudaError_t launch_window_scores_simt(const EvictParams& p, const void* q_win, const void* K,
                                       float* scores, float2* partial, float* rowc,
                                       cudaStream_t s);
@@ -108,6 +115,11 @@ cudaError_t launch_window_combine(const EvictParams& p, const float2* partial, f
                                   cudaStream_t s);
 // Tensor-core scoring path (bf16, d in {64, 128}, G*W <= 256).
 bool window_scores_tc_supported(const EvictParams& p);
+cudaError_t launch_window_votes_tc(const EvictParams& p, const void* q_win, const void* K,
+                                   float* scores, const float* rowc, int32_t* status,
+                                   int32_t* tilectr, cudaStream_t s);
+cudaError_t launch_window_votes_simt(const EvictParams& p, const void* q_win, const void* K,
+                                     float* scores, const float* rowc, cudaStream_t s);
 cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, const void* K,
                                     float* scores, float2* partial, float* rowc, int32_t* status,
                                     int32_t* tilectr, cudaStream_t s);

@@ -5,6 +5,7 @@ never in the CUDA path) and checks that at least one pin then fails: the
 hand-derived closed forms of tests/golden or the brute force.
 """
 import inspect
+import math
 import json
 import os
 import types
@@ -35,6 +36,9 @@ MUTANTS = {
     "decode step over N_kv without the eviction": ("p * ((1.0 - alpha) * n_x + i - 1) + q", "p * (n_x + i - 1) + q"),
     "per-step constant dropped": ("t_decode += p * ((1.0 - alpha) * n_x + i - 1) + q", "t_decode += p * ((1.0 - alpha) * n_x + i - 1)"),
     "pessimistic length rounded down": ("int(min(math.ceil(k * n_hat), n_max))", "int(min(math.floor(k * n_hat), n_max))"),
+    "lse rows see one key too few": ("visible = np.arange(N)[None, :] <= last_seen[:, None]", "visible = np.arange(N)[None, :] < last_seen[:, None]"),
+    "lse without the max added back": ("out[h] = m + np.log(", "out[h] = np.log("),
+    "scores from lse over the window keys too": ("logits = sigma * (q[h] @ k[h // G, :P].T)      # [W][P]\n        S[h // G] += np.exp(logits - L[h][:, None]).sum(axis=0)", "logits = sigma * (q[h] @ k[h // G, 1:P + 1].T)      # [W][P]\n        S[h // G] += np.exp(logits - L[h][:, None]).sum(axis=0)"),
     "predictor overhead ignored": ("return t_predict + wcet(a, b, c, p, q, n_x, al, n_w) - budget", "return wcet(a, b, c, p, q, n_x, al, n_w) - budget"),
     "fit without the constant column": ("for k in range(degree, -1, -1)], axis=1)", "for k in range(degree, 0, -1)], axis=1)"),
     "MAPE relative to the fit": ("np.abs(fit - ta) / ta", "np.abs(fit - ta) / fit"),
@@ -93,6 +97,20 @@ def _pins_pass(m):
         al = m.alpha_star(1e-9, 2e-6, 1e-4, 1e-6, 5e-5, 1000, 10, 1.0, 100, 3e-4, 8e-3, 0.95)
         want = 1.0 - (8e-3 - 3e-4 - (1e-3 + 2e-3 + 1e-4) - 9 * 5e-5 - 36e-6) / 9e-3
         if abs(al - want) > 1e-12 or m.pessimistic_length(10, 1.25, 100) != 13:
+            return False
+        # the window normalisers and the scores rebuilt from them: brute force
+        rng = np.random.default_rng(5)
+        qq, KK2 = rng.standard_normal((4, 5, 8)), rng.standard_normal((2, 23, 8))
+        lse = m.window_lse(qq, KK2)
+        G2 = 2
+        for h in (0, 3):
+            for w in (0, 4):
+                lg = [float(qq[h, w] @ KK2[h // G2, j]) / math.sqrt(8) for j in range(18 + w + 1)]
+                mx = max(lg)
+                if abs(lse[h, w] - (mx + math.log(math.fsum(math.exp(x - mx) for x in lg)))) > 1e-12:
+                    return False
+        if not np.allclose(m.window_scores_from_lse(qq, KK2, lse), np.array(bf.scores(qq.tolist(), KK2.tolist(), G2)),
+                           rtol=1e-12, atol=0):
             return False
         # the least-squares fit: the hand line of tests/test_time_fit.py
         coef, mape = m.fit_time_model([0, 1, 2], [1, 3, 2], 1)
