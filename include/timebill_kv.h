@@ -91,6 +91,21 @@ uint64_t tb_launch_counter(void);
 tb_status tb_retained_count(int64_t n, int32_t window, double alpha,
                             int64_t *k_out, int64_t *r_out);
 
+/* Bits of tb_evict_desc.flags (0 = the default readings). */
+/* Eq. 8 read literally: the retained cache, window included, holds
+ * ceil((1 - alpha) n) rows, so k = that count minus the window, clamped to
+ * [0, n - window] (the window is still always kept). */
+#define TB_EVICT_BUDGET_INCLUDES_WINDOW 1
+/* Average pooling (SnapKV's own pooling) instead of max-pooling: pooled[j] =
+ * (sum of the scores at [j - pool_k/2, j + pool_k/2] inside the prefix) /
+ * pool_k, i.e. out-of-range neighbours count as zeros. */
+#define TB_EVICT_AVG_POOL 2
+
+/* tb_retained_count under the TB_EVICT_BUDGET_INCLUDES_WINDOW bit of
+ * `flags` (other bits are ignored here). Same errors. */
+tb_status tb_retained_count_ex(int64_t n, int32_t window, double alpha,
+                               int32_t flags, int64_t *k_out, int64_t *r_out);
+
 /* Shape of one batched eviction. All pointers are host arrays of length
  * `batch`, read during the call only. */
 typedef struct {
@@ -101,7 +116,7 @@ typedef struct {
   int32_t window;    /* observation window W >= 1 (W <= N_b) */
   int32_t pool_k;    /* max-pool kernel, odd, 1 .. 63 */
   int32_t dtype;     /* tb_dtype of q_win, K, V, Kc, Vc */
-  int32_t reserved;  /* must be 0 */
+  int32_t flags;     /* TB_EVICT_* bits; any other bit is an error */
   const int64_t *n;          /* host [batch]: prompt lengths N_b */
   const double *alpha;       /* host [batch]: eviction ratios in [0, 1] */
   const int64_t *kv_offset;  /* host [batch]: first row of request b in K, V */

@@ -53,6 +53,7 @@ __all__ = [
     "window_lse",
     "window_scores_from_lse",
     "max_pool",
+    "avg_pool",
     "select_indices",
     "gather_rows",
     "score_evict",
@@ -65,7 +66,8 @@ __all__ = [
 ]
 
 
-def retained_count(n: int, window: int, alpha: float) -> Tuple[int, int]:
+def retained_count(n: int, window: int, alpha: float,
+                   budget_includes_window: bool = False) -> Tuple[int, int]:
     """(k, R): retained prefix tokens and retained rows per KV head.
 
     Eq. 8 gives the cache length after evicting a fraction alpha of the N
@@ -74,6 +76,9 @@ def retained_count(n: int, window: int, alpha: float) -> Tuple[int, int]:
     tokens (so alpha = 0 keeps the whole prompt). The ceiling is taken of
     (1-alpha) N - 1e-9 N so that a decimal alpha whose binary value lands a
     hair above an integer product (alpha=0.3, N=10) rounds as written.
+    With budget_includes_window, Eq. 8 is read literally instead: the whole
+    retained cache, window included, is the ceil((1-alpha) N) rows, so the
+    prefix gets that count less W (still clamped; the window stays).
     """
     n = int(n)
     window = int(window)
@@ -83,6 +88,8 @@ def retained_count(n: int, window: int, alpha: float) -> Tuple[int, int]:
         raise ValueError("alpha must lie in [0, 1]")
     p = n - window
     k = math.ceil((1.0 - alpha) * n - 1e-9 * n)
+    if budget_includes_window:
+        k -= window
     k = min(max(k, 0), p)
     return k, k + window
 
@@ -172,6 +179,23 @@ def max_pool(S: np.ndarray, pool_k: int) -> np.ndarray:
     return out
 
 
+def avg_pool(S: np.ndarray, pool_k: int) -> np.ndarray:
+    """1-D average pool along the last axis (SnapKV's pooling): kernel pool_k
+    (odd), stride 1, same padding with zeros, so every output is the sum of
+    the in-range neighbours divided by pool_k."""
+    if pool_k < 1 or pool_k % 2 == 0:
+        raise ValueError("pool_k must be odd and >= 1")
+    S = np.asarray(S, dtype=np.float64)
+    half = pool_k // 2
+    L = S.shape[-1]
+    pad = np.zeros(S.shape[:-1] + (half,))
+    Z = np.concatenate([pad, S, pad], axis=-1)
+    total = np.zeros_like(S)
+    for t in range(pool_k):
+        total += Z[..., t:t + L]
+    return total / pool_k
+
+
 def select_indices(pooled: np.ndarray, k: int, n: int) -> np.ndarray:
     """Retained positions of one KV head: the k prefix positions with the
     largest pooled score (ties to the lower index), then the window
@@ -190,21 +214,26 @@ def gather_rows(X: np.ndarray, idx: np.ndarray) -> np.ndarray:
 
 def score_evict(q_win: np.ndarray, K: np.ndarray, V: np.ndarray, n: Sequence[int],
                 alpha: Sequence[float], kv_offset: Sequence[int], window: int,
-                pool_k: int, heads: Optional[Sequence[int]] = None) -> List[dict]:
+                pool_k: int, heads: Optional[Sequence[int]] = None, pool: str = "max",
+                budget_includes_window: bool = False) -> List[dict]:
     """The whole eviction for a packed batch.
 
     q_win [B][Hq][W][d]; K, V [Hkv][rows][d] with request b at rows
     kv_offset[b] .. kv_offset[b] + n[b]. Returns, per request, a dict with
     k, R, S [Hkv][P], pooled [Hkv][P], idx [Hkv][R], Kc/Vc [Hkv][R][d]
     (in the input array's dtype). ``heads`` restricts the work to some KV
-    heads (the other rows stay zero / empty).
+    heads (the other rows stay zero / empty). ``pool`` is "max" (the
+    default reading) or "avg"; ``budget_includes_window`` selects the literal
+    reading of Eq. 8 in retained_count.
     """
+    if pool not in ("max", "avg"):
+        raise ValueError("pool must be 'max' or 'avg'")
     out = []
     hkv = K.shape[0]
     G = q_win.shape[1] // hkv
     for b in range(len(n)):
         nb, off = int(n[b]), int(kv_offset[b])
-        k, R = retained_count(nb, window, float(alpha[b]))
+        k, R = retained_count(nb, window, float(alpha[b]), budget_includes_window)
         P = nb - window
         hs = range(hkv) if heads is None else heads
         S = np.zeros((hkv, P))
@@ -215,7 +244,7 @@ def score_evict(q_win: np.ndarray, K: np.ndarray, V: np.ndarray, n: Sequence[int
         for g in hs:
             Kg = K[g:g + 1, off:off + nb]
             S[g] = window_scores(q_win[b, g * G:(g + 1) * G], Kg)[0]
-            pooled[g] = max_pool(S[g], pool_k)
+            pooled[g] = max_pool(S[g], pool_k) if pool == "max" else avg_pool(S[g], pool_k)
             idx[g] = select_indices(pooled[g], k, nb)
             Kc[g] = gather_rows(K[g, off:off + nb], idx[g])
             Vc[g] = gather_rows(V[g, off:off + nb], idx[g])

@@ -20,7 +20,8 @@ __all__ = [
     "TB_ERR_CUDA", "TB_ERR_TIMEOUT", "TB_F32", "TB_BF16", "TB_MAX_BATCH",
     "TbError", "EvictDesc", "DecodeDesc", "library_path", "load",
     "tb_status_string", "tb_abi_version", "tb_last_error_detail", "tb_launch_counter",
-    "tb_retained_count", "tb_evict_layout", "tb_evict_workspace_size",
+    "tb_retained_count", "tb_retained_count_ex", "TB_EVICT_BUDGET_INCLUDES_WINDOW",
+    "TB_EVICT_AVG_POOL", "tb_evict_layout", "tb_evict_workspace_size",
     "tb_window_scores", "tb_window_scores_lse", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
     "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_exp2",
@@ -29,6 +30,7 @@ __all__ = [
 
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
 TB_F32, TB_BF16 = 0, 1
+TB_EVICT_BUDGET_INCLUDES_WINDOW, TB_EVICT_AVG_POOL = 1, 2
 TB_MAX_BATCH = 64
 TB_NOALLOC_SCRATCH_BYTES = 4 << 20
 
@@ -40,7 +42,7 @@ class _EvictDescC(ctypes.Structure):
     _fields_ = [
         ("batch", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
         ("head_dim", ctypes.c_int32), ("window", ctypes.c_int32), ("pool_k", ctypes.c_int32),
-        ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("dtype", ctypes.c_int32), ("flags", ctypes.c_int32),
         ("n", _I64P), ("alpha", _F64P), ("kv_offset", _I64P), ("kv_rows", ctypes.c_int64),
         ("out_offset", _I64P), ("out_cap", _I64P), ("out_rows", ctypes.c_int64),
     ]
@@ -93,6 +95,7 @@ def load():
         "tb_last_error_detail": (ctypes.c_char_p, []),
         "tb_launch_counter": (ctypes.c_uint64, []),
         "tb_retained_count": (I, [ctypes.c_int64, I, ctypes.c_double, _I64P, _I64P]),
+        "tb_retained_count_ex": (I, [ctypes.c_int64, I, ctypes.c_double, I, _I64P, _I64P]),
         "tb_evict_layout": (I, [P, _I64P, _I64P]),
         "tb_evict_workspace_size": (I, [P, ctypes.POINTER(SZ)]),
         "tb_window_scores": (I, [P, P, P, P, P, SZ, P]),
@@ -169,7 +172,7 @@ class EvictDesc:
                  kv_offset: Optional[Sequence[int]] = None, kv_rows: Optional[int] = None,
                  out_offset: Optional[Sequence[int]] = None,
                  out_cap: Optional[Sequence[int]] = None, out_rows: Optional[int] = None,
-                 reserved: int = 0):
+                 flags: int = 0):
         self.n = np.ascontiguousarray(n, dtype=np.int64)
         B = self.n.shape[0]
         self.alpha = np.ascontiguousarray(np.resize(np.asarray(alpha, np.float64), B))
@@ -179,7 +182,8 @@ class EvictDesc:
         if kv_rows is None:
             kv_rows = int(self.n.sum())
         if out_cap is None:
-            out_cap = [tb_retained_count(int(nb), window, float(a))[1] if nb >= window >= 1 and 0 <= a <= 1 else 0
+            out_cap = [tb_retained_count_ex(int(nb), window, float(a), flags)[1]
+                       if nb >= window >= 1 and 0 <= a <= 1 else 0
                        for nb, a in zip(self.n, self.alpha)]
         self.out_cap = np.ascontiguousarray(out_cap, dtype=np.int64)
         if out_offset is None:
@@ -188,10 +192,10 @@ class EvictDesc:
         if out_rows is None:
             out_rows = int((self.out_offset + self.out_cap).max()) if B else 0
         self.hq, self.hkv, self.head_dim, self.window = hq, hkv, head_dim, window
-        self.pool_k, self.dtype = pool_k, dtype
+        self.pool_k, self.dtype, self.flags = pool_k, dtype, int(flags)
         self.kv_rows, self.out_rows = int(kv_rows), int(out_rows)
         self.c = _EvictDescC(
-            B, hq, hkv, head_dim, window, pool_k, dtype, reserved,
+            B, hq, hkv, head_dim, window, pool_k, dtype, int(flags),
             self.n.ctypes.data_as(_I64P), self.alpha.ctypes.data_as(_F64P),
             self.kv_offset.ctypes.data_as(_I64P), self.kv_rows,
             self.out_offset.ctypes.data_as(_I64P), self.out_cap.ctypes.data_as(_I64P),
@@ -252,6 +256,14 @@ def tb_retained_count(n: int, window: int, alpha: float):
     r = ctypes.c_int64()
     _check(load().tb_retained_count(int(n), int(window), float(alpha), ctypes.byref(k), ctypes.byref(r)),
            "tb_retained_count")
+    return k.value, r.value
+
+
+def tb_retained_count_ex(n: int, window: int, alpha: float, flags: int = 0):
+    k = ctypes.c_int64()
+    r = ctypes.c_int64()
+    _check(load().tb_retained_count_ex(int(n), int(window), float(alpha), int(flags), ctypes.byref(k),
+                                       ctypes.byref(r)), "tb_retained_count_ex")
     return k.value, r.value
 
 

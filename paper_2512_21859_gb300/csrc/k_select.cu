@@ -1,7 +1,10 @@
 // Max-pool and per-head top-k selection with ordered compaction.
 //
 // Pool[j] = max of S over [j - pool_k/2, j + pool_k/2] clipped to the prefix
-// (stride 1, out-of-range neighbours ignored). Then, per (request, KV head),
+// (stride 1, out-of-range neighbours ignored), or with TB_EVICT_AVG_POOL the
+// sum over that range / pool_k (out-of-range neighbours count as zeros; the
+// selection ranks the sums, whose order is the averages' order, and only the
+// pooled output is scaled). Then, per (request, KV head),
 // the k largest pooled scores are kept, ties to the lower index, and written
 // in ascending index order followed by the window positions P..N-1.
 //
@@ -28,12 +31,14 @@ __global__ void __launch_bounds__(256) pool_kernel(const __grid_constant__ Evict
   const int b = blockIdx.y, g = blockIdx.z;
   const EvictReq& rq = p.req[b];
   const int P = rq.p, half = p.pool_k / 2;
+  const bool avg = (p.flags & TB_EVICT_AVG_POOL) != 0;
+  const float inv = 1.0f / (float)p.pool_k;
   const size_t base = (size_t)g * p.score_rows + rq.score_off;
   for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < P; j += gridDim.x * blockDim.x) {
     const int lo = max(0, j - half), hi = min(P - 1, j + half);
     float m = scores[base + lo];
-    for (int t = lo + 1; t <= hi; ++t) m = fmaxf(m, scores[base + t]);
-    pooled[base + j] = m;
+    for (int t = lo + 1; t <= hi; ++t) m = avg ? m + scores[base + t] : fmaxf(m, scores[base + t]);
+    pooled[base + j] = avg ? m * inv : m;
   }
 }
 
@@ -189,6 +194,7 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   const int b = seg / p.hkv, g = seg % p.hkv;
   const EvictReq& rq = p.req[b];
   const int P = rq.p, k = rq.k, half = p.pool_k / 2;
+  const bool avg = (p.flags & TB_EVICT_AVG_POOL) != 0;
   const int lo = min(P, rank * slice);
   const int cnt = max(0, min(P, lo + slice) - lo);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -198,15 +204,16 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   if (rank == 0)
     for (int t = tid; t < p.window; t += kCsThreads) out[k + t] = P + t;
 
-  // slice + halo, -inf outside the prefix (scores are >= 0, so max is exact);
-  // four loads in flight per thread
+  // slice + halo, -inf outside the prefix for max-pooling (scores are >= 0,
+  // so max is exact), 0 for average pooling; four loads in flight per thread
+  const float pad = avg ? 0.f : -INFINITY;
   const int nin = cnt + 2 * half;
   for (int i0 = tid; i0 < nin; i0 += 4 * kCsThreads) {
     float x[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int i = i0 + q * kCsThreads, j = lo - half + i;
-      x[q] = (i < nin && j >= 0 && j < P) ? S[j] : -INFINITY;
+      x[q] = (i < nin && j >= 0 && j < P) ? S[j] : pad;
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -217,7 +224,7 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   __syncthreads();
   constexpr int kMaxPer = kClusterSliceMax / kCsThreads;
   unsigned reg[kMaxPer];
-  if (half == 3) {  // pool_k = 7: the window as compile-time loads
+  if (half == 3 && !avg) {  // pool_k = 7: the window as compile-time loads
 #pragma unroll
     for (int r = 0; r < kMaxPer; ++r) {
       const int i = tid + r * kCsThreads;
@@ -227,13 +234,22 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
                                        fmaxf(fmaxf(x[4], x[5]), x[6])));
       }
     }
+  } else if (half == 3) {  // the same window, summed in a fixed order
+#pragma unroll
+    for (int r = 0; r < kMaxPer; ++r) {
+      const int i = tid + r * kCsThreads;
+      if (i < cnt) {
+        const float* x = keys_f + i;
+        reg[r] = __float_as_uint(((x[0] + x[1]) + (x[2] + x[3])) + ((x[4] + x[5]) + x[6]));
+      }
+    }
   } else {
 #pragma unroll
     for (int r = 0; r < kMaxPer; ++r) {
       const int i = tid + r * kCsThreads;
       if (i < cnt) {
         float m = keys_f[i];
-        for (int t = 1; t <= 2 * half; ++t) m = fmaxf(m, keys_f[i + t]);
+        for (int t = 1; t <= 2 * half; ++t) m = avg ? m + keys_f[i + t] : fmaxf(m, keys_f[i + t]);
         reg[r] = __float_as_uint(m);
       }
     }
@@ -247,7 +263,8 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   __syncthreads();
   if (pooled_out) {
     float* po = pooled_out + (size_t)g * p.score_rows + rq.score_off + lo;
-    for (int i = tid; i < cnt; i += kCsThreads) po[i] = __uint_as_float(keys[i]);
+    const float scale = avg ? 1.0f / (float)p.pool_k : 1.0f;
+    for (int i = tid; i < cnt; i += kCsThreads) po[i] = __uint_as_float(keys[i]) * scale;
   }
 
   // ---- radix select of the k-th largest key (uniform across the cluster)

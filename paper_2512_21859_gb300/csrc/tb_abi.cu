@@ -34,11 +34,12 @@ namespace {
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // k = ceil((1 - alpha) n - 1e-9 n), clamped to [0, n - window] (Eq. 8 reading).
-bool retained(int64_t n, int32_t window, double alpha, int64_t* k, int64_t* r) {
+bool retained(int64_t n, int32_t window, double alpha, int32_t flags, int64_t* k, int64_t* r) {
   if (window < 1 || n < window) return false;
   if (!(alpha >= 0.0 && alpha <= 1.0)) return false;
   const double x = (1.0 - alpha) * (double)n - 1e-9 * (double)n;
   int64_t kk = (int64_t)ceil(x);
+  if (flags & TB_EVICT_BUDGET_INCLUDES_WINDOW) kk -= window;
   const int64_t p = n - window;
   if (kk < 0) kk = 0;
   if (kk > p) kk = p;
@@ -57,7 +58,8 @@ bool ranges_overlap(const int64_t* off, const int64_t* len, int batch) {
 
 tb_status build_evict(const tb_evict_desc* d, EvictParams* p) {
   if (!d) return TB_ERR_INVALID_ARG;
-  if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->window < 1 || d->reserved != 0)
+  if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->window < 1 ||
+      (d->flags & ~(TB_EVICT_BUDGET_INCLUDES_WINDOW | TB_EVICT_AVG_POOL)) != 0)
     return TB_ERR_INVALID_ARG;
   if (d->batch > TB_MAX_BATCH) return TB_ERR_UNSUPPORTED;
   if (d->hq % d->hkv != 0) return TB_ERR_INVALID_ARG;
@@ -79,6 +81,7 @@ tb_status build_evict(const tb_evict_desc* d, EvictParams* p) {
   p->d = d->head_dim;
   p->window = d->window;
   p->pool_k = d->pool_k;
+  p->flags = d->flags;
   p->dtype = d->dtype;
   p->m_rows = (int32_t)m_rows;
   p->chunk = kSimtChunk;
@@ -93,7 +96,7 @@ tb_status build_evict(const tb_evict_desc* d, EvictParams* p) {
     const int64_t n = d->n[b];
     if (n < d->window || n > (int64_t(1) << 30)) return TB_ERR_INVALID_ARG;
     int64_t k, r;
-    if (!retained(n, d->window, d->alpha[b], &k, &r)) return TB_ERR_INVALID_ARG;
+    if (!retained(n, d->window, d->alpha[b], d->flags, &k, &r)) return TB_ERR_INVALID_ARG;
     if (d->kv_offset[b] < 0 || d->kv_offset[b] + n > d->kv_rows) return TB_ERR_INVALID_ARG;
     if (d->out_offset[b] < 0 || d->out_cap[b] < r ||
         d->out_offset[b] + d->out_cap[b] > d->out_rows)
@@ -305,9 +308,14 @@ uint64_t tb_launch_counter(void) { return g_launches.load(std::memory_order_rela
 
 tb_status tb_retained_count(int64_t n, int32_t window, double alpha, int64_t* k_out,
                             int64_t* r_out) {
+  return tb_retained_count_ex(n, window, alpha, 0, k_out, r_out);
+}
+
+tb_status tb_retained_count_ex(int64_t n, int32_t window, double alpha, int32_t flags,
+                               int64_t* k_out, int64_t* r_out) {
   if (!k_out || !r_out) return TB_ERR_INVALID_ARG;
   int64_t k, r;
-  if (!retained(n, window, alpha, &k, &r)) return TB_ERR_INVALID_ARG;
+  if (!retained(n, window, alpha, flags, &k, &r)) return TB_ERR_INVALID_ARG;
   *k_out = k;
   *r_out = r;
   return TB_OK;

@@ -45,7 +45,7 @@ struct EvictParams {
   int32_t items;      // total scoring work items
   int32_t max_p;      // max_b P_b
   int32_t max_r;      // max_b R_b
-  int32_t pad0;
+  int32_t flags;      // TB_EVICT_* bits of the descriptor
   int64_t kv_rows, out_rows, score_rows, idx_rows;
   float scale_log2;   // log2(e) / sqrt(d)
   float rowc_scale;   // c_row = rowc[r] * rowc_scale in log2 units: 1 for the

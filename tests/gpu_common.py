@@ -24,19 +24,20 @@ def from_dev(t, dtype: str) -> np.ndarray:
     return t.cpu().numpy()
 
 
-def evict_desc(wl, lay, extra_cap: int = 0):
+def evict_desc(wl, lay, extra_cap: int = 0, flags: int = 0):
     n, a = lay["n"], lay["alpha"]
-    caps = [tb.tb_retained_count(int(nb), wl.window, float(ab))[1] + extra_cap for nb, ab in zip(n, a)]
+    caps = [tb.tb_retained_count_ex(int(nb), wl.window, float(ab), flags)[1] + extra_cap
+            for nb, ab in zip(n, a)]
     return tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, window=wl.window,
                         pool_k=wl.pool_k, dtype=DT[wl.dtype], n=n, alpha=a,
-                        kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)), out_cap=caps)
+                        kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)), out_cap=caps, flags=flags)
 
 
-def run_evict(wl, lay, extra_cap: int = 0, dev=None):
+def run_evict(wl, lay, extra_cap: int = 0, dev=None, flags: int = 0):
     """tb_score_evict on the GPU; returns host copies of idx, pooled, Kc, Vc and the
     device tensors (for decode)."""
     import torch
-    desc = evict_desc(wl, lay, extra_cap)
+    desc = evict_desc(wl, lay, extra_cap, flags)
     if dev is None:
         dev = {k: to_dev(lay[k], wl.dtype) for k in ("q_win", "K", "V")}
     score_rows, idx_rows = tb.tb_evict_layout(desc)
@@ -57,7 +58,8 @@ def run_evict(wl, lay, extra_cap: int = 0, dev=None):
 def request_slices(desc, b):
     """(score column offset, idx column offset) of request b."""
     P = [int(n) - desc.window for n in desc.n]
-    R = [tb.tb_retained_count(int(n), desc.window, float(a))[1] for n, a in zip(desc.n, desc.alpha)]
+    R = [tb.tb_retained_count_ex(int(n), desc.window, float(a), desc.flags)[1]
+         for n, a in zip(desc.n, desc.alpha)]
     return int(np.sum(P[:b])), int(np.sum(R[:b])), P[b], R[b]
 
 

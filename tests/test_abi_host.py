@@ -95,7 +95,7 @@ def test_layout_and_workspace(tb):
     (dict(kv_offset=[-1]), 1),
     (dict(out_cap=[100]), 1),                # out_cap < R
     (dict(out_rows=10), 1),
-    (dict(reserved=1), 1),
+    (dict(flags=4), 1),                      # a flag bit the library does not know
     (dict(n=[512] * 65, alpha=[0.5] * 65), 2),  # batch > TB_MAX_BATCH
     (dict(hq=2048, hkv=1), 2),               # G*W beyond the supported window rows
 ])

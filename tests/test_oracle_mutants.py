@@ -39,6 +39,9 @@ MUTANTS = {
     "lse rows see one key too few": ("visible = np.arange(N)[None, :] <= last_seen[:, None]", "visible = np.arange(N)[None, :] < last_seen[:, None]"),
     "lse without the max added back": ("out[h] = m + np.log(", "out[h] = np.log("),
     "scores from lse over the window keys too": ("logits = sigma * (q[h] @ k[h // G, :P].T)      # [W][P]\n        S[h // G] += np.exp(logits - L[h][:, None]).sum(axis=0)", "logits = sigma * (q[h] @ k[h // G, 1:P + 1].T)      # [W][P]\n        S[h // G] += np.exp(logits - L[h][:, None]).sum(axis=0)"),
+    "avg pool over the in-range count": ("    return total / pool_k\n", "    return total / np.convolve(np.ones(L), np.ones(pool_k), 'same')\n"),
+    "avg pool one narrower": ("    for t in range(pool_k):\n        total += Z[..., t:t + L]", "    for t in range(pool_k - 1):\n        total += Z[..., t:t + L]"),
+    "literal budget keeps the window on top": ("        k -= window\n", "        k -= 0\n"),
     "predictor overhead ignored": ("return t_predict + wcet(a, b, c, p, q, n_x, al, n_w) - budget", "return wcet(a, b, c, p, q, n_x, al, n_w) - budget"),
     "fit without the constant column": ("for k in range(degree, -1, -1)], axis=1)", "for k in range(degree, 0, -1)], axis=1)"),
     "MAPE relative to the fit": ("np.abs(fit - ta) / ta", "np.abs(fit - ta) / fit"),
@@ -111,6 +114,12 @@ def _pins_pass(m):
                     return False
         if not np.allclose(m.window_scores_from_lse(qq, KK2, lse), np.array(bf.scores(qq.tolist(), KK2.tolist(), G2)),
                            rtol=1e-12, atol=0):
+            return False
+        # the eviction variants: the literal Eq. 8 budget and the average pool
+        if m.retained_count(100, 16, 0.5, budget_includes_window=True) != (34, 50):
+            return False
+        ap = m.avg_pool(np.full(12, 2.0), 7)
+        if not (np.allclose(ap[3:9], 2.0) and np.allclose(ap[:3], 2.0 * np.array([4, 5, 6]) / 7)):
             return False
         # the least-squares fit: the hand line of tests/test_time_fit.py
         coef, mape = m.fit_time_model([0, 1, 2], [1, 3, 2], 1)
