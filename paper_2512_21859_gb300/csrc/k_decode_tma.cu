@@ -139,6 +139,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_barrier_init();
   }
   __syncthreads();
+  // everything above touched only shared memory and kernel parameters
+  pdl_wait();
+  pdl_trigger();
 
   auto issue = [&](int t) {
     const int s = t % kStages;
@@ -483,8 +486,9 @@ cudaError_t launch_g(const DecodeParams& p, const CUtensorMap& tk, const CUtenso
   auto kern = decode_tma<D, G>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
-  kern<<<dim3(p.splits, p.hkv, p.batch), kThreads, Gm::kSmem, s>>>(
-      p, tk, tv, static_cast<const uint16_t*>(q), lens, part_o, part_ml, counters, out, status);
+  e = launch_pdl(kern, dim3(p.splits, p.hkv, p.batch), dim3(kThreads), Gm::kSmem, s, p, tk, tv,
+                 static_cast<const uint16_t*>(q), lens, part_o, part_ml, counters, out, status);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

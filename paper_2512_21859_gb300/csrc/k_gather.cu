@@ -26,6 +26,8 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(
   constexpr int kVecs = kRowsPerWarp * 2 * VPR;  // vectors a warp moves
   constexpr int kPerLane = kVecs / 32;
   static_assert(kPerLane <= kMaxVecPerLane, "too many vectors per lane");
+  pdl_wait();  // idx comes from the select kernel just before
+  pdl_trigger();
   const int b = blockIdx.y, g = blockIdx.z;
   const EvictReq& rq = p.req[b];
   const int R = rq.k + p.window;
@@ -74,13 +76,15 @@ cudaError_t launch_gather(const EvictParams& p, const int32_t* idx, const void* 
   const uint4* v4 = static_cast<const uint4*>(V);
   uint4* kc4 = static_cast<uint4*>(Kc);
   uint4* vc4 = static_cast<uint4*>(Vc);
+  cudaError_t e;
   switch (vec_per_row) {
-    case 8: gather_kernel<8><<<grid, kGatherThreads, 0, s>>>(p, idx, k4, v4, kc4, vc4); break;
-    case 16: gather_kernel<16><<<grid, kGatherThreads, 0, s>>>(p, idx, k4, v4, kc4, vc4); break;
-    case 32: gather_kernel<32><<<grid, kGatherThreads, 0, s>>>(p, idx, k4, v4, kc4, vc4); break;
+    case 8: e = launch_pdl(gather_kernel<8>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4); break;
+    case 16: e = launch_pdl(gather_kernel<16>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4); break;
+    case 32: e = launch_pdl(gather_kernel<32>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4); break;
     default: return cudaErrorInvalidValue;
   }
   count_launches(1);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

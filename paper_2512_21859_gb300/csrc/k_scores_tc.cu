@@ -278,6 +278,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
+  // (no early pdl_trigger here: the select's CTAs launched during the scoring
+  // made the 128K step ~2 us slower on GB300; the select starts on completion)
   const uint32_t tmem = bars->tmem_base;
   volatile int* abort = &bars->abort;
   int issued = 0, committed = 0;

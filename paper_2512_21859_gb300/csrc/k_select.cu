@@ -198,6 +198,8 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   const int lo = min(P, rank * slice);
   const int cnt = max(0, min(P, lo + slice) - lo);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  pdl_wait();  // the scores come from the kernel just before
+  pdl_trigger();
   const float* S = scores + (size_t)g * p.score_rows + rq.score_off;
   int32_t* out = idx + (size_t)g * p.idx_rows + rq.idx_off;
 
@@ -467,13 +469,15 @@ cudaError_t launch_select_cluster(const EvictParams& p, const float* scores, flo
   cfg.blockDim = dim3(kCsThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (unsigned)cs;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;
   e = cudaLaunchKernelEx(&cfg, select_cluster_kernel, p, scores, pooled_out, idx, slice);
   count_launches(1);
   if (e != cudaSuccess) return e;

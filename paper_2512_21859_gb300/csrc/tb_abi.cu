@@ -6,6 +6,7 @@
 
 #include <cmath>
 #include <math.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <algorithm>
@@ -244,12 +245,19 @@ tb_status run_select(const EvictParams& p, const EvictWorkspace& w, const float*
 
 void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
 
+bool pdl_enabled() {
+  static const bool on = getenv("TB_NO_PDL") == nullptr;
+  return on;
+}
+
 namespace {
 
 // Clears a workspace's control words (status word, split / tile counters)
 // ahead of the call's kernels. A kernel node costs about a fifth of what a
 // memset node does inside a CUDA graph (~0.7 vs ~3.5 us between kernels).
 __global__ void clear_words(uint4* __restrict__ w, size_t n16) {
+  pdl_wait();
+  pdl_trigger();
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16;
        i += (size_t)gridDim.x * blockDim.x)
     w[i] = make_uint4(0u, 0u, 0u, 0u);
@@ -261,8 +269,10 @@ cudaError_t clear_control_words(void* ws, size_t bytes, cudaStream_t s) {
   const size_t n16 = bytes / 16;  // callers pass multiples of 256 bytes
   if (n16 == 0) return cudaSuccess;
   const unsigned blocks = (unsigned)std::min<size_t>((n16 + 255) / 256, 152);
-  clear_words<<<blocks, 256, 0, s>>>(static_cast<uint4*>(ws), n16);
+  const cudaError_t e =
+      launch_pdl(clear_words, dim3(blocks), dim3(256), 0, s, static_cast<uint4*>(ws), n16);
   count_launches(1);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

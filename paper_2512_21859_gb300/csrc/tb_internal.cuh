@@ -92,6 +92,36 @@ bool make_bf16_map(CUtensorMap* map, const void* base, int d, uint64_t rows, int
 // Adds n to the process-wide launch counter (tb_launch_counter).
 void count_launches(int n);
 
+// Programmatic dependent launch. A kernel launched by launch_pdl may begin
+// (its CTAs made resident, their set-up run) while the previous kernel of the
+// stream is still finishing: it calls pdl_wait() before its first access to
+// global memory, which returns once that kernel has completed and its writes
+// are visible, and pdl_trigger() after it, which lets the next such launch
+// start early. Both are no-ops for a kernel launched the ordinary way.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// False when the environment sets TB_NO_PDL (ordinary launches throughout).
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
+}
+
 // Zeroes the first `bytes` (a multiple of 16) of a workspace on stream s
 // with one small kernel.
 cudaError_t clear_control_words(void* ws, size_t bytes, cudaStream_t s);
