@@ -24,6 +24,12 @@
  *    Every device pointer must be 16-byte aligned.
  *  - No exceptions cross the ABI; every call returns a tb_status.
  *  - Calls that share a workspace must not overlap on the GPU.
+ *  - The decode, select, gather and workspace-clearing kernels are launched
+ *    with programmatic dependent launch: each may be scheduled while the
+ *    kernel before it in the stream finishes, and waits for that kernel's
+ *    completion before it touches global memory, so stream order holds as
+ *    usual. Setting the environment variable TB_NO_PDL (read once per
+ *    process) launches them the ordinary way.
  *
  * Notation: B requests; request b has prompt length N_b, eviction ratio
  * alpha_b and P_b = N_b - W prefix tokens (the last W prompt tokens form the
