@@ -54,6 +54,8 @@ def parse_args(argv=None):
     ap.add_argument("--sweep", default=None,
                     help="comma-separated alphas: print one line per alpha")
     ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--no-variants", action="store_true",
+                    help="skip timing tb_window_scores_lse beside the step (its line is then null)")
     ap.add_argument("--fit-time-model", action="store_true",
                     help="profile tb_decode_attn over N_kv and tb_score_evict over N_x on the 7b "
                          "shape and print the least-squares time model (Eq. 6a/6b) with its MAPE")
@@ -377,7 +379,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                      "alg_flops_per_launch": t["flops"],
                      "flops_rule": "2 Hq W d flops per key and pass: N keys (statistics) + N - W keys (sums)", "hbm_frac": sroof[dom]["frac"]})
 
-    lse_var = time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, ms_step, n, peaks)
+    lse_var = None if args.no_variants else time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers,
+                                                             stage_ms, ms_step, n, peaks)
 
     e2e = run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R)
 
