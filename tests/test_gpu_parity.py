@@ -217,20 +217,34 @@ def test_shapes(case):
 # stages alone, bit-exact on oracle-produced inputs
 # ---------------------------------------------------------------------------
 
-@pytest.mark.parametrize("seed", [0, 1, 2])
-def test_select_stage_exact_on_oracle_scores(seed):
+@pytest.mark.parametrize("seed,values", [(0, "grid64"), (1, "grid64"), (2, "grid64"),
+                                         (3, "mant12"), (4, "cont"), (5, "mant12")])
+def test_select_stage_exact_on_oracle_scores(seed, values):
+    """grid64: multiples of 1/64 (ties everywhere); mant12: 12 significant
+    bits, so the threshold value recurs ~50 times among 100K keys and is
+    resolved among gathered candidates after three radix digits; cont:
+    continuous values, resolved among candidates after two digits."""
     rng = np.random.default_rng(seed)
     W, pk = 16, 7
     ns = [int(x) for x in rng.integers(W, 20000, size=5)] + [W, W + 1]
     alphas = list(rng.uniform(0, 1, size=len(ns)))
     alphas[0] = 0.0
     alphas[1] = 1.0
+    if values != "grid64":   # two long prefixes (8-CTA clusters) with a partial selection
+        ns = [100_000, 65_000] + ns[:3]
+        alphas = [0.9, 0.5] + alphas[:3]
     hkv = 3
     desc = tb.EvictDesc(hq=hkv, hkv=hkv, head_dim=64, window=W, pool_k=pk, dtype=tb.TB_F32,
                         n=ns, alpha=alphas)
     score_rows, idx_rows = tb.tb_evict_layout(desc)
-    # scores with many exact ties (quantised) and a heavy tail
-    S = (np.floor(rng.exponential(1.0, size=(hkv, max(score_rows, 1))) * 64) / 64).astype(np.float32)
+    shape = (hkv, max(score_rows, 1))
+    if values == "grid64":   # many exact ties (quantised) and a heavy tail
+        S = (np.floor(rng.exponential(1.0, size=shape) * 64) / 64).astype(np.float32)
+    elif values == "mant12":
+        x = 1.0 + rng.random(shape)
+        S = (np.round(x * 2048) / 2048).astype(np.float32)
+    else:
+        S = (rng.exponential(1.0, size=shape) ** 3 * 1e-3).astype(np.float32)
     S_t = torch.from_numpy(S).cuda()
     idx = torch.full((hkv, idx_rows), -1, dtype=torch.int32, device="cuda")
     pooled = torch.zeros_like(S_t)
