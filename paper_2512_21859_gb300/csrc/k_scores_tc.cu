@@ -474,8 +474,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     if (MODE == kPassBoth) {
-      // publish this CTA's partials, then meet the grid (one thread waits)
-      __threadfence();
+      // publish this CTA's partials, then meet the grid (one thread waits).
+      // The writers need no fence of their own: __syncwarp orders each lane's
+      // writes before lane 0's arrive (a CTA-scope release), the waiter's
+      // acquire then precedes its GPU-scope fence and arrival, and that
+      // release is cumulative over everything ordered before it.
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->pub);
       if (warp == 0 && lane == 0) {
