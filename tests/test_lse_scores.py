@@ -143,3 +143,36 @@ def test_gpu_lse_rejects_bad_pointers():
     with pytest.raises(tb.TbError) as e:
         tb.tb_window_scores_lse(desc, q, K, None, S, ws)
     assert e.value.status == tb.TB_ERR_INVALID_ARG
+
+
+@pytest.mark.gpu
+def test_gpu_lse_128k_sampled_heads():
+    """The one-pass call at the full 128K size the benchmark times
+    (32q/8kv, N 131072, W 64): KV heads 0 and 7 recomputed by the oracle from
+    the same fp32 normalisers; the other heads get finite stand-ins."""
+    torch, tb = _gpu()
+    from tests.gpu_common import to_dev
+    wl = inputs.WORKLOADS["128k"]
+    lay = inputs.make_layer(wl, 0)
+    n = int(lay["n"][0])
+    q = inputs.as_f32(lay["q_win"], "bf16")
+    K = inputs.as_f32(lay["K"], "bf16")
+    G = wl.group
+    lse = np.zeros((1, wl.hq, wl.window), dtype=np.float32)
+    heads = (0, 7)
+    for g in heads:
+        lse[0, g * G:(g + 1) * G] = orc.window_lse(q[0, g * G:(g + 1) * G], K[g:g + 1, :n]).astype(np.float32)
+    desc = tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, window=wl.window, pool_k=wl.pool_k,
+                        dtype=tb.TB_BF16, n=lay["n"], alpha=lay["alpha"])
+    score_rows, _ = tb.tb_evict_layout(desc)
+    scores = torch.zeros((wl.hkv, score_rows), dtype=torch.float32, device="cuda")
+    ws = torch.empty(tb.tb_evict_workspace_size(desc), dtype=torch.uint8, device="cuda")
+    tb.tb_window_scores_lse(desc, to_dev(lay["q_win"], "bf16"), to_dev(lay["K"], "bf16"),
+                            torch.from_numpy(lse).cuda(), scores, ws)
+    st, raw = tb.tb_read_status(ws)
+    assert st == tb.TB_OK, raw
+    got = scores.cpu().numpy()
+    for g in heads:
+        ref = orc.window_scores_from_lse(q[0, g * G:(g + 1) * G], K[g:g + 1, :n],
+                                         lse[0, g * G:(g + 1) * G].astype(np.float64))
+        np.testing.assert_allclose(got[g], ref[0], rtol=3e-6, atol=0)
