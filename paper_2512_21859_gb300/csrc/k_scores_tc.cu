@@ -248,9 +248,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const size_t segrow = ((size_t)info.b * p.hkv + info.g) * M;
 
-  if (MODE == kPassVotes)
-    for (int r = threadIdx.x; r < 256; r += blockDim.x)
-      ncr[r] = r < M ? -(rowc[segrow + r] * p.rowc_scale) : -INFINITY;
 
   // ---- set-up: barriers and the TMEM allocation
   if (threadIdx.x == 0) {
@@ -278,6 +275,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
+  // global memory from here on (the votes-only launch is a programmatic
+  // dependent launch: its set-up above overlapped the previous kernel)
+  pdl_wait();
+  if (MODE == kPassVotes) {
+    for (int r = threadIdx.x; r < 256; r += blockDim.x)
+      ncr[r] = r < M ? -(rowc[segrow + r] * p.rowc_scale) : -INFINITY;
+    __syncthreads();
+  }
   // (no early pdl_trigger here: the select's CTAs launched during the scoring
   // made the 128K step ~2 us slower on GB300; the select starts on completion)
   const uint32_t tmem = bars->tmem_base;
@@ -774,9 +779,10 @@ cudaError_t launch_window_votes_tc(const EvictParams& p, const void* q_win, cons
   auto launch = [&](auto kern, int smem) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    kern<<<pt.items, kThreads, smem, s>>>(pt, tq, tk, nullptr, rowc, scores, status, gsync,
-                                           tilectr);
+    e = launch_pdl(kern, dim3(pt.items), dim3(kThreads), smem, s, pt, tq, tk, (float2*)nullptr, rowc,
+                   scores, status, gsync, tilectr);
     count_launches(1);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
   };
   return p.d == 64 ? launch(ws_tc<64, kPassVotes>, Geo<64>::kSmem)
