@@ -59,8 +59,19 @@ constexpr int kBoxBytes = 128 * 128;  // one TMA box: 128 rows x 64 bf16
 // bound by streaming K, and the epilogue by latency, not by MUFU throughput),
 // so all of them use MUFU.
 constexpr int kMufuElems = 32;
+// Set in the grid-barrier word when a row maximum is too large for the fp64
+// row sums (those heads then merge their partials the slow way).
+constexpr uint32_t kSumOverflowBit = 0x80000000u;
+// When some head is scored by more CTAs than this, the fused kernel sums its
+// rows' (max, sum) partials in fp64 atomically as pass 1 ends (the kRowSums
+// instantiation), so that after the grid barrier c_row is one load per row
+// instead of a merge over every chunk. Measured on GB300: with 37 chunks per
+// head (32K) the scoring took 26.4 -> 24.2 us; with 19 (128K) it did not pay.
+constexpr int kSumMinChunks = 24;
 
-enum : int { kPassStats = 1, kPassVotes = 2, kPassBoth = 3 };
+// kRowSums (with kPassBoth): the fp64 row sums replace the post-barrier
+// merge; a separate instantiation, so the kernel without it is unchanged
+enum : int { kPassStats = 1, kPassVotes = 2, kPassBoth = 3, kRowSums = 4 };
 
 template <int D>
 struct Geo {
@@ -93,6 +104,7 @@ struct Bars {
   int abort;
   int codes[8];   // tile code of the it-th tile the producer claimed, at [it % 8]
   int accode[2];  // the MMA warp's copy for the accumulator it fills
+  int sums_ok;    // kRowSums: every row's fp64 sum is usable (no row max beyond the range)
 };
 
 // Tile codes: t >= 0 is pass 1 tile t, -2 - t is pass 2 tile t, kNoTile ends.
@@ -221,7 +233,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     ws_tc(const __grid_constant__ EvictParams p, const __grid_constant__ CUtensorMap tq,
           const __grid_constant__ CUtensorMap tk, float2* __restrict__ partial,
           const float* __restrict__ rowc, float* __restrict__ scores, int32_t* __restrict__ status,
-          uint32_t* __restrict__ gsync, int32_t* __restrict__ tilectr) {
+          uint32_t* __restrict__ gsync, int32_t* __restrict__ tilectr,
+          double* __restrict__ lsum) {
   using G = Geo<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
@@ -247,6 +260,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int NP = (M + 15) & ~15;   // pass 2 MMA N: window rows rounded up to 16
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const size_t segrow = ((size_t)info.b * p.hkv + info.g) * M;
+  constexpr bool kFused = (MODE & kPassBoth) == kPassBoth;
+  constexpr bool kSums = kFused && (MODE & kRowSums) != 0;
 
 
   // ---- set-up: barriers and the TMEM allocation
@@ -474,11 +489,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float l =
               (m == -INFINITY) ? 0.f : l_run * fast_exp2(m_run - m) + o.y * fast_exp2(o.x - m);
           partial[(size_t)item * M + row] = make_float2(m, l);
+          if (kSums && l > 0.f) {
+            // the row's sum over the whole grid, sum_c l_c 2^(m_c), in fp64 (no
+            // common reference needed: 2^m stays finite for |m| < 960, which
+            // leaves room for the sum); larger rows take the slow merge
+            if (fabsf(m) < 960.f) {
+              // l 2^m = (l 2^f) 2^i with m = i + f, f in [0, 1): the fp32
+              // factors multiply exactly in fp64, the power of two is a scale
+              const float fi = floorf(m);
+              const double two_i = __longlong_as_double((long long)(1023 + (int)fi) << 52);
+              atomicAdd(&lsum[segrow + row], (double)l * (double)exp2f(m - fi) * two_i);
+            } else {
+              atomicOr(gsync, kSumOverflowBit);  // read with the barrier count
+            }
+          }
         }
       }
     }
 
-    if (MODE == kPassBoth) {
+    if (kFused) {
       // publish this CTA's partials, then meet the grid (one thread waits).
       // The writers need no fence of their own: __syncwarp orders each lane's
       // writes before lane 0's arrive (a CTA-scope release), the waiter's
@@ -491,7 +520,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           __threadfence();
           atomicAdd(gsync, 1u);
           const uint64_t t0 = tc::globaltimer();
-          while (ld_acquire(gsync) < gridDim.x) {
+          uint32_t seen;
+          while (((seen = ld_acquire(gsync)) & (kSums ? ~kSumOverflowBit : ~0u)) < gridDim.x) {
             if (*abort) break;
             if (tc::globaltimer() - t0 > tc::kWaitNs) {
               *abort = 1;
@@ -500,12 +530,29 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             __nanosleep(64);
           }
+          if (kSums) bars->sums_ok = (seen & kSumOverflowBit) == 0;
         }
         tc::mbar_arrive(&bars->gready);  // also on abort: the waiters then see the flag
       }
       ok = ok && tc::mbar_wait(&bars->gready, 0, abort, status) && !*abort;
-      // merge every chunk of this (request, KV head) into -c_row
-      if (ok) {
+      // -c_row of every window row: log2 of its fp64 grid sum, or, when a row
+      // maximum was out of that range, the merge of every chunk's partial
+      if (kSums && ok && bars->sums_ok) {
+        if (threadIdx.x < 256) {
+          const int r = threadIdx.x;
+          float v = -INFINITY;
+          if (r < M) {
+            // log2 of the fp64 sum: its binary exponent plus log2 of the
+            // mantissa in [1, 2), the latter in fp32
+            const long long bits = __double_as_longlong(__ldcg(&lsum[segrow + r]));
+            const int e = (int)((bits >> 52) & 0x7ff) - 1023;
+            const float mant = (float)__longlong_as_double((bits & 0x000fffffffffffffLL) |
+                                                           0x3ff0000000000000LL);
+            v = -((float)e + log2f(mant));
+          }
+          ncr[r] = v;
+        }
+      } else if (ok) {
         const size_t it0 = (size_t)rq.item0 + (size_t)info.g * info.nch;
         // two threads per window row (adjacent lanes) fold alternate CTAs'
         // partials in one pass (online rescaling, compensated sums), then
@@ -670,10 +717,10 @@ int coresident_ctas(const void* kernel, int smem, int slot) {
 template <int D>
 cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const CUtensorMap& tk,
                             float* scores, float2* partial, float* rowc, int32_t* status,
-                            int32_t* tilectr, cudaStream_t s) {
+                            int32_t* tilectr, double* lsum, cudaStream_t s) {
   using Gm = Geo<D>;
   uint32_t* gsync = reinterpret_cast<uint32_t*>(status) + kGridSyncWord;
-  auto fused = ws_tc<D, kPassBoth>;
+  auto fused = window_scores_row_sums(pt) ? ws_tc<D, kPassBoth | kRowSums> : ws_tc<D, kPassBoth>;
   cudaError_t e =
       cudaFuncSetAttribute(fused, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
@@ -689,7 +736,7 @@ cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const 
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, fused, pt, tq, tk, partial, (const float*)rowc, scores, status,
-                           gsync, tilectr);
+                           gsync, tilectr, lsum);
     count_launches(1);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
@@ -702,11 +749,11 @@ cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const 
   e = cudaFuncSetAttribute(votes, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
   stats<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync,
-                                              tilectr);
+                                              tilectr, (double*)nullptr);
   e = launch_window_combine(pt, partial, rowc, s);
   if (e != cudaSuccess) return e;
   votes<<<pt.items, kThreads, Gm::kSmem, s>>>(pt, tq, tk, partial, rowc, scores, status, gsync,
-                                              tilectr);
+                                              tilectr, (double*)nullptr);
   count_launches(2);
   return cudaGetLastError();
 }
@@ -755,15 +802,16 @@ EvictParams tc_item_params(const EvictParams& p) {
 
 cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, const void* K,
                                     float* scores, float2* partial, float* rowc, int32_t* status,
-                                    int32_t* tilectr, cudaStream_t s) {
+                                    int32_t* tilectr, double* lsum, cudaStream_t s) {
   const EvictParams pt = tc_item_params(p);
   CUtensorMap tq, tk;
   const uint64_t qrows = (uint64_t)p.batch * p.hq * p.window;
   const uint64_t krows = (uint64_t)p.hkv * p.kv_rows;
   if (!make_bf16_map(&tq, q_win, p.d, qrows, 128) || !make_bf16_map(&tk, K, p.d, krows, 128))
     return cudaErrorInvalidValue;
-  return p.d == 64 ? launch_tc_typed<64>(pt, tq, tk, scores, partial, rowc, status, tilectr, s)
-                   : launch_tc_typed<128>(pt, tq, tk, scores, partial, rowc, status, tilectr, s);
+  return p.d == 64
+             ? launch_tc_typed<64>(pt, tq, tk, scores, partial, rowc, status, tilectr, lsum, s)
+             : launch_tc_typed<128>(pt, tq, tk, scores, partial, rowc, status, tilectr, lsum, s);
 }
 
 cudaError_t launch_window_votes_tc(const EvictParams& p, const void* q_win, const void* K,
@@ -780,13 +828,21 @@ cudaError_t launch_window_votes_tc(const EvictParams& p, const void* q_win, cons
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     e = launch_pdl(kern, dim3(pt.items), dim3(kThreads), smem, s, pt, tq, tk, (float2*)nullptr, rowc,
-                   scores, status, gsync, tilectr);
+                   scores, status, gsync, tilectr, (double*)nullptr);
     count_launches(1);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   };
   return p.d == 64 ? launch(ws_tc<64, kPassVotes>, Geo<64>::kSmem)
                    : launch(ws_tc<128, kPassVotes>, Geo<128>::kSmem);
+}
+
+bool window_scores_row_sums(const EvictParams& p) {
+  if (!window_scores_tc_supported(p)) return false;
+  const EvictParams pt = tc_item_params(p);
+  for (int b = 0; b < p.batch; ++b)
+    if ((p.req[b].n + pt.chunk - 1) / pt.chunk > kSumMinChunks) return true;
+  return false;
 }
 
 }  // namespace tb

@@ -133,6 +133,8 @@ EvictWorkspace carve_evict(const EvictParams& p) {
   off += kStatusBytes;
   w.tilectr = off;
   off = align_up(off + 2 * sizeof(int32_t) * (size_t)p.batch * p.hkv, 256);
+  w.lsum = off;
+  off = align_up(off + sizeof(double) * (size_t)p.batch * p.hkv * p.m_rows, 256);
   w.zeroed = off;
   w.scores = off;
   off = align_up(off + sizeof(float) * (size_t)p.hkv * p.score_rows, 256);
@@ -225,11 +227,17 @@ T* at(void* base, size_t off) {
   return reinterpret_cast<T*>(static_cast<char*>(base) + off);
 }
 
+// The control words every eviction call clears: the status area and the
+// tile counters, and the fp64 row sums when the scoring kernel uses them.
+size_t evict_clear_bytes(const EvictParams& p, const EvictWorkspace& w) {
+  return window_scores_row_sums(p) ? w.zeroed : w.lsum;
+}
+
 tb_status run_window_scores(const EvictParams& p, const EvictWorkspace& w, const void* q_win,
                             const void* K, float* scores, void* ws, cudaStream_t s) {
   return cuda_status(launch_window_scores(p, q_win, K, scores, at<float2>(ws, w.partial),
                                           at<float>(ws, w.rowc), at<int32_t>(ws, w.status),
-                                          at<int32_t>(ws, w.tilectr), s));
+                                          at<int32_t>(ws, w.tilectr), at<double>(ws, w.lsum), s));
 }
 
 tb_status run_select(const EvictParams& p, const EvictWorkspace& w, const float* scores,
@@ -286,9 +294,9 @@ cudaError_t launch_window_votes(const EvictParams& p, const void* q_win, const v
 
 cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
                                  float* scores, float2* partial, float* rowc, int32_t* status,
-                                 int32_t* tilectr, cudaStream_t s) {
+                                 int32_t* tilectr, double* lsum, cudaStream_t s) {
   if (window_scores_tc_supported(p))
-    return launch_window_scores_tc(p, q_win, K, scores, partial, rowc, status, tilectr, s);
+    return launch_window_scores_tc(p, q_win, K, scores, partial, rowc, status, tilectr, lsum, s);
   return launch_window_scores_simt(p, q_win, K, scores, partial, rowc, s);
 }
 
@@ -486,7 +494,7 @@ tb_status tb_window_scores(const tb_evict_desc* desc, const void* q_win, const v
   const EvictWorkspace w = carve_evict(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(clear_control_words(workspace, w.zeroed, s))) != TB_OK) return st;
+  if ((st = cuda_status(clear_control_words(workspace, evict_clear_bytes(p, w), s))) != TB_OK) return st;
   return run_window_scores(p, w, q_win, K, scores, workspace, s);
 }
 
@@ -502,7 +510,7 @@ tb_status tb_window_scores_lse(const tb_evict_desc* desc, const void* q_win, con
   const EvictWorkspace w = carve_evict(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(clear_control_words(workspace, w.zeroed, s))) != TB_OK) return st;
+  if ((st = cuda_status(clear_control_words(workspace, evict_clear_bytes(p, w), s))) != TB_OK) return st;
   p.rowc_scale = 1.4426950408889634f;  // natural-log LSE -> log2 units
   return cuda_status(launch_window_votes(p, q_win, K, scores, lse, at<int32_t>(workspace, w.status),
                                          at<int32_t>(workspace, w.tilectr), s));
@@ -549,7 +557,7 @@ tb_status tb_score_evict(const tb_evict_desc* desc, const void* q_win, const voi
   const EvictWorkspace w = carve_evict(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(clear_control_words(workspace, w.zeroed, s))) != TB_OK) return st;
+  if ((st = cuda_status(clear_control_words(workspace, evict_clear_bytes(p, w), s))) != TB_OK) return st;
   float* scores = at<float>(workspace, w.scores);
   if ((st = run_window_scores(p, w, q_win, K, scores, workspace, s)) != TB_OK) return st;
   if ((st = run_select(p, w, scores, idx, pooled, workspace, s)) != TB_OK) return st;

@@ -21,6 +21,7 @@ enum : int32_t {
 constexpr size_t kStatusBytes = 256;
 constexpr int kGridSyncWord = 16;
 
+
 // Largest G*W (window rows of one KV-head group) the scoring kernels take.
 constexpr int kMaxWindowRows = 1024;
 
@@ -80,9 +81,10 @@ tb_status cuda_status(cudaError_t e);
 
 // Workspace carving for the eviction calls (byte offsets, 256-aligned).
 // status: kStatusBytes; tilectr: two tile counters per (request, KV head) of
-// the tensor-core scoring kernel; [0, zeroed) is cleared by every call.
+// the tensor-core scoring kernel; lsum: fp64 row sums sum_c l_c 2^(m_c) of
+// its window rows; [0, zeroed) is cleared by every call.
 struct EvictWorkspace {
-  size_t status, tilectr, zeroed, scores, partial, rowc, pooled, total;
+  size_t status, tilectr, lsum, zeroed, scores, partial, rowc, pooled, total;
 };
 
 // 2-D bf16 TMA map over rows of d elements, boxes of box_rows x 64 columns
@@ -131,7 +133,7 @@ cudaError_t clear_control_words(void* ws, size_t bytes, cudaStream_t s);
 // ---------------------------------------------------------------------------
 cudaError_t launch_window_scores(const EvictParams& p, const void* q_win, const void* K,
                                  float* scores, float2* partial, float* rowc,
-                                 int32_t* status, int32_t* tilectr, cudaStream_t s);
+                                 int32_t* status, int32_t* tilectr, double* lsum, cudaStream_t s);
 // The normalised window sums alone, from given per-row log2-sum-exp values
 // (rowc [B][Hkv][G*W], scaled by p.rowc_scale): one QK^T pass.
 cudaError_t launch_window_votes(const EvictParams& p, const void* q_win, const void* K,
@@ -145,6 +147,9 @@ cudaError_t launch_window_combine(const EvictParams& p, const float2* partial, f
                                   cudaStream_t s);
 // Tensor-core scoring path (bf16, d in {64, 128}, G*W <= 256).
 bool window_scores_tc_supported(const EvictParams& p);
+// Whether the scoring kernel uses the fp64 row sums (workspace `lsum`) for
+// some (request, KV head) of this descriptor; they are cleared only then.
+bool window_scores_row_sums(const EvictParams& p);
 cudaError_t launch_window_votes_tc(const EvictParams& p, const void* q_win, const void* K,
                                    float* scores, const float* rowc, int32_t* status,
                                    int32_t* tilectr, cudaStream_t s);
@@ -152,7 +157,7 @@ cudaError_t launch_window_votes_simt(const EvictParams& p, const void* q_win, co
                                      float* scores, const float* rowc, cudaStream_t s);
 cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, const void* K,
                                     float* scores, float2* partial, float* rowc, int32_t* status,
-                                    int32_t* tilectr, cudaStream_t s);
+                                    int32_t* tilectr, double* lsum, cudaStream_t s);
 cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled,
                         cudaStream_t s);
 cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* idx,

@@ -380,3 +380,27 @@ def test_fma_pipe_exp2_against_exact():
     ref = np.exp2(xc)
     rel = np.abs(y - ref) / ref
     assert rel.max() < 2.2e-7, (rel.max(), x[np.argmax(rel)])
+
+
+@pytest.mark.parametrize("big", [False, True])
+def test_many_chunks_per_head_row_sums(big):
+    """One KV head over 32K keys is split across many CTAs, so the scoring
+    kernel takes its fp64 row-sum path for the window statistics; with logits
+    near 700 (big) a row maximum leaves that path's range and the partials
+    are merged instead. Both against the oracle."""
+    rng = np.random.default_rng(77 + big)
+    hq, hkv, d, W, n = 4, 1, 128, 64, 32768
+    base = 8.0 if big else 0.0
+    q = base + rng.standard_normal((1, hq, W, d)).astype(np.float32) * (0.05 if big else 1.0)
+    K = base + rng.standard_normal((hkv, n, d)).astype(np.float32) * (0.05 if big else 1.0 / np.sqrt(d))
+    V = rng.standard_normal((hkv, n, d)).astype(np.float32)
+    lay = {"q_win": inputs.f32_to_bf16(q), "K": inputs.f32_to_bf16(K), "V": inputs.f32_to_bf16(V),
+           "n": np.array([n], dtype=np.int64), "alpha": np.array([0.7]), "kv_offset": np.zeros(1, np.int64)}
+    wl = _custom("bf16", hq, hkv, d, W, 7, seed=0)
+    res = run_evict(wl, lay)
+    ref = _oracle(wl, lay)
+    if big:
+        # the logits this case needs: beyond 960 in log2 units
+        s_max = float(np.max(inputs.as_f32(lay["q_win"], "bf16")[0, 0] @ inputs.as_f32(lay["K"], "bf16")[0, :64].T))
+        assert s_max / np.sqrt(d) * np.log2(np.e) > 960
+    _check_evict(wl, lay, res, ref)
