@@ -427,7 +427,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   // flight together; the first chunk of its first output group is requested
   // before the split weights are computed, so that those loads and the
   // (max, sum) loads travel at once.
-  constexpr int kChunk = 16;
+  // (one chunk covers the ~38 splits per thread of one request with four KV
+  // heads; with NS > 1 each thread has about half as many)
+  constexpr int kChunk = NS >= 2 ? 16 : 40;
   float4 ov[kChunk];
   {
     const int e0 = tid, e = e0 / NS, part = e0 % NS;
