@@ -242,13 +242,45 @@ tb_status tb_decode_attn(const tb_decode_desc *desc, const void *q,
                          tb_stream_t stream);
 
 /*
+ * tb_decode_attn for a decode loop that keeps its workspace from step to
+ * step (the paper has no counterpart: a deployment fast path). tb_decode_attn
+ * zeroes the workspace's control words (status word, split counters) with a
+ * small kernel before every step, which on GB300 costs about 1 us per call
+ * between the previous kernel and this one; this entry point launches only
+ * the decode kernel.
+ *  - tb_decode_workspace_prepare zeroes the control words of a workspace of
+ *    at least tb_decode_workspace_size bytes for `desc`; call it once after
+ *    allocating the workspace (and again after any error or status flag).
+ *    A workspace prepared for one descriptor serves every descriptor whose
+ *    tb_decode_workspace_size is no larger and whose batch and hkv are the
+ *    same (the split counters are indexed by request and KV head).
+ *  - tb_decode_attn_prepared computes exactly what tb_decode_attn computes,
+ *    with the same arguments; each call leaves the split counters at zero
+ *    when it completes. The status word is not cleared between calls: a
+ *    flag (a length above its cap, a bounded wait that gave up) stays set
+ *    until the workspace is prepared again.
+ *  - Calls sharing one workspace must not overlap on the GPU (one stream, or
+ *    ordered by events), as for tb_decode_attn.
+ * Errors: as tb_decode_attn.
+ */
+tb_status tb_decode_workspace_prepare(const tb_decode_desc *desc,
+                                      void *workspace, size_t workspace_bytes,
+                                      tb_stream_t stream);
+tb_status tb_decode_attn_prepared(const tb_decode_desc *desc, const void *q,
+                                  const void *Kc, const void *Vc,
+                                  const int32_t *lens, void *out,
+                                  void *workspace, size_t workspace_bytes,
+                                  tb_stream_t stream);
+
+/*
  * Waits for `stream`, then reads the status word kept at the start of a
  * workspace used by the calls above: TB_OK, TB_ERR_TIMEOUT (a bounded
  * device-side wait gave up) or TB_ERR_INVALID_ARG (a device-side range check
  * fired, e.g. a decode length above its cap). *raw (if not NULL) receives the
  * word itself. The word is cleared at the start of every call that can set
  * it: tb_window_scores, tb_score_evict and tb_decode_attn (tb_select_topk
- * and tb_gather_kv never set it and leave it as it was).
+ * and tb_gather_kv never set it and leave it as it was;
+ * tb_decode_attn_prepared keeps it until tb_decode_workspace_prepare).
  */
 tb_status tb_read_status(const void *workspace, size_t workspace_bytes,
                          tb_stream_t stream, int32_t *raw);

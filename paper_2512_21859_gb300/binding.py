@@ -25,6 +25,7 @@ __all__ = [
     "tb_window_scores", "tb_window_scores_lse", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
     "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_exp2",
+    "tb_decode_workspace_prepare", "tb_decode_attn_prepared",
     "TimeModel", "tb_wcet", "tb_alpha_star", "tb_fit_time_model",
 ]
 
@@ -107,6 +108,8 @@ def load():
         "tb_decode_attn": (I, [P, P, P, P, P, P, P, SZ, P]),
         "tb_read_status": (I, [P, SZ, P, ctypes.POINTER(I)]),
         "tb_decode_attn_noalloc": (I, [P, P, P, P, P, P, P]),
+        "tb_decode_workspace_prepare": (I, [P, P, SZ, P]),
+        "tb_decode_attn_prepared": (I, [P, P, P, P, P, P, P, SZ, P]),
         "tb_diag_exp2": (I, [P, P, ctypes.c_int64, P]),
         "tb_wcet": (I, [P, ctypes.c_int64, ctypes.c_double, ctypes.c_int64, ctypes.POINTER(ctypes.c_double)]),
         "tb_alpha_star": (I, [P, ctypes.c_int64, ctypes.c_double, ctypes.c_double, ctypes.c_int64,
@@ -328,6 +331,23 @@ def tb_decode_attn(desc: DecodeDesc, q, Kc, Vc, lens, out, workspace, workspace_
     w, wb = _ws(workspace, workspace_bytes)
     _check(load().tb_decode_attn(desc.ref(), _ptr(q), _ptr(Kc), _ptr(Vc), _ptr(lens), _ptr(out), w, wb,
                                  _stream(stream)), "tb_decode_attn")
+
+
+def tb_decode_workspace_prepare(desc: DecodeDesc, workspace, workspace_bytes=None, stream=None):
+    """Zeroes a decode workspace's control words once, for tb_decode_attn_prepared."""
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_decode_workspace_prepare(desc.ref(), w, wb, _stream(stream)),
+           "tb_decode_workspace_prepare")
+
+
+def tb_decode_attn_prepared(desc: DecodeDesc, q, Kc, Vc, lens, out, workspace, workspace_bytes=None,
+                            stream=None):
+    """tb_decode_attn without the per-call clearing kernel, on a workspace that
+    tb_decode_workspace_prepare zeroed once (its status word then stays set
+    until the next prepare)."""
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_decode_attn_prepared(desc.ref(), _ptr(q), _ptr(Kc), _ptr(Vc), _ptr(lens), _ptr(out),
+                                          w, wb, _stream(stream)), "tb_decode_attn_prepared")
 
 
 def tb_decode_attn_noalloc(desc: DecodeDesc, q, Kc, Vc, lens, out, stream=None):

@@ -149,22 +149,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::tma_load_2d(st + (Gm::KH + h) * kBox, &tv, h * 64, row0 + t * kTile, &full[s]);
     }
   };
-  // The first tiles are requested before the dependency wait. The kernel
-  // launched just before this one on the stream is always the library's own
-  // clearing kernel (it writes only the workspace's control words), which
-  // lets this one start only after its own wait has returned, i.e. once every
-  // earlier kernel has completed and its writes are visible; the cache rows
-  // cannot be written by the clearing kernel. On GB300 the requests so moved
-  // ahead the first tile's arrival by 0.2-0.7 us per call.
+  // With p.early_tma the first tiles are requested before the dependency
+  // wait: the kernel launched just before this one on the stream is then the
+  // library's own clearing kernel (it writes only the workspace's control
+  // words), which lets this one start only after its own wait has returned,
+  // i.e. once every earlier kernel has completed and its writes are visible;
+  // the cache rows cannot be written by the clearing kernel. Without it (a
+  // prepared workspace, no clearing kernel) any kernel may precede this one,
+  // so the requests wait for it.
   int issued = 0;
   if (tid == 0) {
     tc::tma_prefetch_desc(&tk);
     tc::tma_prefetch_desc(&tv);
-    for (; issued < kStages && issued < ntiles_c; ++issued) issue(issued);
+    if (p.early_tma)
+      for (; issued < kStages && issued < ntiles_c; ++issued) issue(issued);
   }
-  // everything below may touch what the clearing kernel writes
   pdl_wait();
   pdl_trigger();
+  if (tid == 0)
+    for (; issued < kStages && issued < ntiles_c; ++issued) issue(issued);
   int len = lens[b];
   if (len > (int)cap64) {
     if (split == 0 && g == 0 && tid == 0) atomicOr(status, kStatusRange);
@@ -411,6 +414,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                  : "l"(counters + b * p.hkv + g)
                  : "memory");
     *last_flag = prev == p.splits - 1;
+    // every split has counted in: the counter goes back to zero for the next
+    // call (what a prepared workspace relies on; the clearing kernel of the
+    // other entry points zeroes it anyway)
+    if (*last_flag) counters[b * p.hkv + g] = 0;
   }
   __syncthreads();
   if (!*last_flag) return;

@@ -202,6 +202,7 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
   splits = (d->max_len + split_len - 1) / split_len;
   p->splits = (int32_t)splits;
   p->split_len = (int32_t)split_len;
+  p->early_tma = 1;
   return TB_OK;
 }
 
@@ -590,6 +591,39 @@ tb_status tb_decode_attn(const tb_decode_desc* desc, const void* q, const void* 
                                    at<float2>(workspace, w.part_ml),
                                    at<int32_t>(workspace, w.counters),
                                    at<int32_t>(workspace, w.status), s));
+}
+
+tb_status tb_decode_workspace_prepare(const tb_decode_desc* desc, void* workspace,
+                                      size_t workspace_bytes, tb_stream_t stream) {
+  DecodeParams p;
+  tb_status st = build_decode(desc, &p);
+  if (st != TB_OK) return st;
+  const DecodeWorkspace w = carve_decode(p);
+  if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
+  return cuda_status(
+      clear_control_words(workspace, w.part_o, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+tb_status tb_decode_attn_prepared(const tb_decode_desc* desc, const void* q, const void* Kc,
+                                  const void* Vc, const int32_t* lens, void* out, void* workspace,
+                                  size_t workspace_bytes, tb_stream_t stream) {
+  DecodeParams p;
+  tb_status st = build_decode(desc, &p);
+  if (st != TB_OK) return st;
+  if (!q || !Kc || !Vc || !lens || !out) return TB_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(Kc) || !aligned16(Vc) || !aligned16(out))
+    return TB_ERR_INVALID_ARG;
+  const DecodeWorkspace w = carve_decode(p);
+  if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
+  // no clearing kernel: the split counters are zero since the workspace was
+  // prepared (each call's last split CTA zeroes its counter again), and the
+  // status word keeps what earlier calls raised
+  p.early_tma = 0;
+  return cuda_status(launch_decode(p, q, Kc, Vc, lens, out, at<float>(workspace, w.part_o),
+                                   at<float2>(workspace, w.part_ml),
+                                   at<int32_t>(workspace, w.counters),
+                                   at<int32_t>(workspace, w.status),
+                                   reinterpret_cast<cudaStream_t>(stream)));
 }
 
 tb_status tb_read_status(const void* workspace, size_t workspace_bytes, tb_stream_t stream,

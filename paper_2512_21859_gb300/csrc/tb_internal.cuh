@@ -58,7 +58,10 @@ struct EvictParams {
 struct DecodeParams {
   int32_t batch, hq, hkv, group, d, dtype, out_dtype, splits;
   int32_t split_len;  // keys per split
-  int32_t pad0;
+  // 1: the kernel just before the decode on the stream is the library's own
+  // clearing kernel, so the first K/V tiles may be requested before the
+  // dependency wait; 0 (prepared workspaces): anything may precede it
+  int32_t early_tma;
   int64_t cache_rows;
   int64_t max_len;
   float scale_log2;

@@ -178,3 +178,21 @@ def test_decode_call_fails_before_launch(tb):
     with pytest.raises(tb.TbError) as e:
         tb.tb_decode_attn(d, fake, fake, fake, fake, fake, fake, wb - 1, stream=0)
     assert e.value.status == tb.TB_ERR_WORKSPACE
+
+
+def test_prepared_decode_calls_fail_before_launch(tb):
+    d = _ddesc(tb)
+    wb = tb.tb_decode_workspace_size(d)
+    fake = 1 << 20
+    with pytest.raises(tb.TbError) as e:
+        tb.tb_decode_attn_prepared(d, fake, fake, fake, 0, fake, fake, wb, stream=0)
+    assert e.value.status == tb.TB_ERR_INVALID_ARG
+    with pytest.raises(tb.TbError) as e:
+        tb.tb_decode_attn_prepared(d, fake, fake, fake, fake, fake, fake, wb - 1, stream=0)
+    assert e.value.status == tb.TB_ERR_WORKSPACE
+    with pytest.raises(tb.TbError) as e:
+        tb.tb_decode_workspace_prepare(d, fake, wb - 1, stream=0)
+    assert e.value.status == tb.TB_ERR_WORKSPACE
+    with pytest.raises(tb.TbError) as e:
+        tb.tb_decode_workspace_prepare(_ddesc(tb, hq=30), fake, wb, stream=0)
+    assert e.value.status == tb.TB_ERR_INVALID_ARG
