@@ -185,7 +185,7 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   namespace cg = cooperative_groups;
   cg::cluster_group cluster = cg::this_cluster();
   __shared__ ClusterSelectShared sh;
-  extern __shared__ float keys_f[];  // slice + 2 * halo floats
+  extern __shared__ __align__(16) float keys_f[];  // slice + 2 * halo floats (+ slack)
   unsigned* keys = reinterpret_cast<unsigned*>(keys_f);
 
   const int cs = (int)cluster.num_blocks();
@@ -226,14 +226,29 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   __syncthreads();
   constexpr int kMaxPer = kClusterSliceMax / kCsThreads;
   unsigned reg[kMaxPer];
-  if (half == 3 && !avg) {  // pool_k = 7: the window as compile-time loads
+  // pool_k = 7, max: each thread pools groups of four consecutive outputs
+  // 4q .. 4q+3 from the ten inputs keys_f[4q .. 4q+9], read as three 16-byte
+  // vectors (the smem array has slack past its inputs for the last group's
+  // vectors; values there only reach outputs >= cnt, which are not kept).
+  // Three vector loads per four outputs instead of seven scalar loads per
+  // output: the pooling is bound by shared-memory wavefronts.
+  const bool grouped = half == 3 && !avg;
+  if (grouped) {
 #pragma unroll
-    for (int r = 0; r < kMaxPer; ++r) {
-      const int i = tid + r * kCsThreads;
-      if (i < cnt) {
-        const float* x = keys_f + i;
-        reg[r] = __float_as_uint(fmaxf(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])),
-                                       fmaxf(fmaxf(x[4], x[5]), x[6])));
+    for (int r = 0; r < kMaxPer / 4; ++r) {
+      const int q = tid + r * kCsThreads;
+      if (4 * q < cnt) {
+        const float4 u = *reinterpret_cast<const float4*>(keys_f + 4 * q);
+        const float4 v = *reinterpret_cast<const float4*>(keys_f + 4 * q + 4);
+        const float4 w = *reinterpret_cast<const float4*>(keys_f + 4 * q + 8);
+        // inputs x0..x9 = u.x u.y u.z u.w v.x v.y v.z v.w w.x w.y; output k is
+        // the max of x_k .. x_{k+6}, all four share x3..x6
+        const float core = fmaxf(fmaxf(u.w, v.x), fmaxf(v.y, v.z));
+        const float m12 = fmaxf(u.y, u.z), m78 = fmaxf(v.w, w.x);
+        reg[4 * r + 0] = __float_as_uint(fmaxf(fmaxf(core, u.x), m12));
+        reg[4 * r + 1] = __float_as_uint(fmaxf(fmaxf(core, m12), v.w));
+        reg[4 * r + 2] = __float_as_uint(fmaxf(fmaxf(core, u.z), m78));
+        reg[4 * r + 3] = __float_as_uint(fmaxf(fmaxf(core, m78), w.y));
       }
     }
   } else if (half == 3) {  // the same window, summed in a fixed order
@@ -257,10 +272,25 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
     }
   }
   __syncthreads();
+  if (grouped) {
 #pragma unroll
-  for (int r = 0; r < kMaxPer; ++r) {
-    const int i = tid + r * kCsThreads;
-    if (i < cnt) keys[i] = reg[r];
+    for (int r = 0; r < kMaxPer / 4; ++r) {
+      const int q = tid + r * kCsThreads;
+      if (4 * q + 3 < cnt) {
+        *reinterpret_cast<uint4*>(keys + 4 * q) =
+            make_uint4(reg[4 * r], reg[4 * r + 1], reg[4 * r + 2], reg[4 * r + 3]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          if (4 * q + k < cnt) keys[4 * q + k] = reg[4 * r + k];
+      }
+    }
+  } else {
+#pragma unroll
+    for (int r = 0; r < kMaxPer; ++r) {
+      const int i = tid + r * kCsThreads;
+      if (i < cnt) keys[i] = reg[r];
+    }
   }
   __syncthreads();
   if (pooled_out) {
@@ -460,7 +490,8 @@ cudaError_t launch_select_cluster(const EvictParams& p, const float* scores, flo
                                   int32_t* idx, cudaStream_t s) {
   const int cs = select_cluster_size(p);
   const int slice = (p.max_p + cs - 1) / cs;
-  const size_t smem = sizeof(float) * ((size_t)slice + 2 * (p.pool_k / 2));
+  // slice + halo, plus slack for the grouped max-pool's last 16-byte loads
+  const size_t smem = sizeof(float) * (((size_t)slice + 2 * (p.pool_k / 2) + 8 + 3) & ~(size_t)3);
   cudaError_t e = cudaFuncSetAttribute(select_cluster_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
