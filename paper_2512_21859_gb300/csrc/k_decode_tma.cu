@@ -5,7 +5,7 @@
 // softmax over the request's first len keys, attention definition of
 // "FLOPs-based Modeling"), organised for HBM bandwidth: each CTA takes one
 // (request, KV head, key split) and streams its K and V rows through a
-// 6-stage ring of 64-key tiles that one thread fills with 2-D TMA copies
+// 3-stage ring of 128-key tiles that one thread fills with 2-D TMA copies
 // (128-byte swizzle, so ldmatrix reads are free of bank conflicts). The G
 // query heads of the group share every tile, so each K/V byte is read from
 // HBM once per decode step.
@@ -18,10 +18,11 @@
 //   O += P V       P in fp32 is split into a bf16 part and a bf16 residual,
 //                  both multiplied by V (ldmatrix.trans) and accumulated in
 //                  fp32, so P enters with ~16 significant bits.
-// At the end the four warps merge in shared memory into the split's partial
+// At the end the eight warps merge in shared memory into the split's partial
 // (max, sum, unnormalised output); the CTA that finishes last among a
-// (request, KV head)'s splits (a counter in the workspace, zeroed by every
-// call) merges the splits and writes the output.
+// (request, KV head)'s splits (a counter in the workspace: zero before the
+// call, and set back to zero by that CTA) merges the splits and writes the
+// output.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -338,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
 
-  // ---- merge the four warps: O, m, l through shared memory (the ring is free)
+  // ---- merge the eight warps: O, m, l through shared memory (the ring is free)
 #pragma unroll
   for (int hr = 0; hr < 2; ++hr) {
     l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 1);

@@ -240,8 +240,9 @@ __device__ __forceinline__ uint64_t sub2(uint64_t a, uint64_t b) {
   return d;
 }
 
-// 2^x for a pair of x <= ~0.5 on the FMA pipes instead of the MUFU unit (which
-// issues 16 exponentials per SM per clock). Cody-Waite split x = n + f with n
+// 2^x for a pair of x <= ~0.5 on the FMA pipes instead of the MUFU unit (about
+// 32 exponentials per SM per clock on GB300, as ncu's XU-pipe counts of the
+// scoring kernel put it). Cody-Waite split x = n + f with n
 // = round(x) (by adding 1.5 * 2^23) and f in [-0.5, 0.5]; 2^f by a degree-5
 // polynomial fitted for minimum relative error (exp2_poly_fit.py: 2.1e-7 in
 // fp32); 2^n added to the exponent field. x is clamped at -125 so that the
