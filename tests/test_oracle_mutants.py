@@ -15,7 +15,7 @@ import pytest
 
 from oracle import timebill_oracle as orc
 from tests import brute_force as bf
-from tests.test_oracle_pins import GOLDEN, _frac_expr, _golden_vote_inputs
+from tests.test_oracle_pins import GOLDEN, _frac_expr, _golden_vote_inputs, _packed_decode_case
 
 SRC = inspect.getsource(orc)
 
@@ -32,6 +32,10 @@ MUTANTS = {
     "budget counts the window inside": ("return k, k + window", "return max(k - window, 0), max(k - window, 0) + window"),
     "decode scale dropped": ("s = sigma * (kk @ q[h])", "s = kk @ q[h]"),
     "decode attends one row too many": ("kk = np.asarray(Kc[g, :length]", "kk = np.asarray(Kc[g, :length + 1]"),
+    "packed decode slices one row late": ("Kc[:, off:off + L], Vc[:, off:off + L]", "Kc[:, off + 1:off + 1 + L], Vc[:, off + 1:off + 1 + L]"),
+    "packed decode reads the next request's offset": ("off, L = int(cache_offset[b]), int(lens[b])", "off, L = int(cache_offset[min(b + 1, B - 1)]), int(lens[b])"),
+    "packed decode writes the wrong request": ("        out[b] = decode_attention(q[b]", "        out[B - 1 - b] = decode_attention(q[b]"),
+    "packed decode takes one request's length for all": ("off, L = int(cache_offset[b]), int(lens[b])", "off, L = int(cache_offset[b]), int(lens[0])"),
     "decoding steps counted from i = 0": ("for i in range(1, n_w):", "for i in range(0, n_w):"),
     "decode step over N_kv without the eviction": ("p * ((1.0 - alpha) * n_x + i - 1) + q", "p * (n_x + i - 1) + q"),
     "per-step constant dropped": ("t_decode += p * ((1.0 - alpha) * n_x + i - 1) + q", "t_decode += p * ((1.0 - alpha) * n_x + i - 1)"),
@@ -96,6 +100,15 @@ def _pins_pass(m):
         ref = bf.attention(qq[0, 0].tolist(), KK[0].tolist(), VV[0].tolist(), 20)
         if not np.allclose(out[0], ref, rtol=1e-12):
             return False
+        # the packed-batch decode against the brute force on unpacked caches
+        qb, caches, Kp, Vp, lens, offs, Gb = _packed_decode_case()
+        ob = m.decode_batch(qb, Kp, Vp, lens, offs)
+        for b, (Kb, Vb) in enumerate(caches):
+            for h in (0, qb.shape[1] - 1):
+                want = [0.0] * qb.shape[2] if lens[b] == 0 else bf.attention(
+                    qb[b, h].tolist(), Kb[h // Gb].tolist(), Vb[h // Gb].tolist(), lens[b])
+                if not np.allclose(ob[b, h], want, rtol=1e-12, atol=1e-14):
+                    return False
         # the budgeted eviction ratio: the hand example of tests/test_alpha_star.py
         al = m.alpha_star(1e-9, 2e-6, 1e-4, 1e-6, 5e-5, 1000, 10, 1.0, 100, 3e-4, 8e-3, 0.95)
         want = 1.0 - (8e-3 - 3e-4 - (1e-3 + 2e-3 + 1e-4) - 9 * 5e-5 - 36e-6) / 9e-3

@@ -326,3 +326,51 @@ def test_decode_invariances():
     np.testing.assert_allclose(orc.decode_attention(q, Kc, Vc, 1), np.tile(Vc[0, 0], (2, 1)))
     # a convex combination of the values
     assert np.all(base <= Vc[0].max(axis=0) + 1e-12) and np.all(base >= Vc[0].min(axis=0) - 1e-12)
+
+
+# --------------------------------------------------------------------------
+# The packed-batch decode the GPU parity tests compare against
+# --------------------------------------------------------------------------
+
+def _packed_decode_case(seed=21):
+    """Four requests whose caches are drawn first as separate arrays and
+    only then packed at non-contiguous row offsets, with filler rows (huge
+    values) between and after them, so that a wrong offset or a wrong
+    request index changes the result."""
+    rng = np.random.default_rng(seed)
+    hkv, G, d = 2, 3, 5
+    lens = [7, 0, 12, 1]
+    caps = [9, 3, 14, 4]
+    caches = [(rng.standard_normal((hkv, c, d)), rng.standard_normal((hkv, c, d))) for c in caps]
+    q = rng.standard_normal((len(lens), hkv * G, d))
+    gaps = [2, 1, 5, 3]
+    offs, rows = [], 0
+    for c, gap in zip(caps, gaps):
+        rows += gap
+        offs.append(rows)
+        rows += c
+    Kp = np.full((hkv, rows + 2, d), 1e3)
+    Vp = np.full((hkv, rows + 2, d), -1e3)
+    for (Kb, Vb), o, c in zip(caches, offs, caps):
+        Kp[:, o:o + c] = Kb
+        Vp[:, o:o + c] = Vb
+    return q, caches, Kp, Vp, lens, offs, G
+
+
+def test_decode_batch_matches_unpacked_brute_force():
+    q, caches, Kp, Vp, lens, offs, G = _packed_decode_case()
+    out = orc.decode_batch(q, Kp, Vp, lens, offs)
+    assert out.shape == q.shape
+    for b, (Kb, Vb) in enumerate(caches):
+        for h in range(q.shape[1]):
+            g = h // G
+            if lens[b] == 0:
+                assert np.all(out[b, h] == 0.0)
+                continue
+            ref = bf.attention(q[b, h].tolist(), Kb[g].tolist(), Vb[g].tolist(), lens[b])
+            np.testing.assert_allclose(out[b, h], ref, rtol=1e-12, atol=1e-14)
+    # one request alone through the single-request routine on its own arrays
+    Kb, Vb = caches[2]
+    np.testing.assert_allclose(out[2], orc.decode_attention(q[2], Kb, Vb, lens[2]), rtol=1e-13)
+    # a length-1 request returns its first value row, its heads' own group
+    np.testing.assert_allclose(out[3], np.repeat(caches[3][1][:, 0], G, axis=0), rtol=1e-13)
