@@ -42,6 +42,15 @@ from paper_2512_21859_gb300 import inputs  # noqa: E402
 METRIC = "evict + decode-attn µs/layer and HBM GB/s (fraction of ~8 TB/s) vs α"
 L2_BYTES = 129e6
 NOMINAL_HBM_GBS = 8000.0
+# the metric's alpha axis, carried in the one JSON line of every run
+ALPHA_SWEEP = [("128k", (0.5, 0.75, 0.9)), ("32k", (0.0, 0.25, 0.5, 0.75, 0.9, 0.95))]
+# the algorithmic bytes of each stage per launch (the method's minimum)
+SURVEY_BYTES_RULE = {
+    "window_scores": "e Hkv d sum(N) + q_win bytes: K read once",
+    "select_topk": "4 Hkv (2 sum(P) + sum(R)): scores read, pooled written, indices written",
+    "gather_kv": "4 e Hkv d sum(R): retained K and V rows read and written",
+    "decode_attn": "2 e Hkv d sum(len) + B Hq d (e + 4): compacted K and V read, query read, fp32 output",
+}
 
 
 def parse_args(argv=None):
@@ -62,6 +71,10 @@ def parse_args(argv=None):
                     help="profile tb_decode_attn_prepared over N_kv and tb_score_evict over N_x on the 7b "
                          "shape and print the least-squares time model (Eq. 6a/6b) with its MAPE")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-alpha-sweep", action="store_true",
+                    help="skip the per-alpha stage table (128K at 0.5/0.75/0.9, 32K at 0..0.95)")
+    ap.add_argument("--sweep-steps", type=int, default=12,
+                    help="launches per stage timing of each alpha point")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target seconds of oracle work for the cpu_baseline sample")
     return ap.parse_args(argv)
@@ -98,11 +111,14 @@ def alg_bytes(wl, n, alpha, lens):
 
 
 def stage_rooflines(wl, n, ab, stage_ms, peaks):
-    """Every stage against its roofline: algorithmic bytes over the stage time
-    against the measured copy bandwidth; the window scoring also as a tensor
-    contraction (2 Hq W d flops per key and pass; pass 1 over the N keys,
-    pass 2 over the P = N - W prefix keys) against the
-    measured sustained bf16 rate (its kernel runs inside a long step)."""
+    """Every stage against its HBM roofline: algorithmic bytes over the
+    stage's per-launch time against the measured copy bandwidth. The window
+    scoring is also a dense bf16 contraction; beside its HBM fraction it
+    reports the tensor rate on the method's flops (one Q K^T over the N keys
+    of every window row, 2 Hq W d N) and on the flops this kernel executes
+    (two passes: N keys for the row statistics, then the P = N - W prefix
+    keys for the sums), both against the measured burst bf16 rate (the
+    stage is timed alone, in graphs of a few hundred microseconds)."""
     hbm = float(peaks["hbm_gbs"])
     out = {}
     for s, ms in stage_ms.items():
@@ -110,12 +126,19 @@ def stage_rooflines(wl, n, ab, stage_ms, peaks):
         out[s] = {"bound": "hbm", "alg_bytes": int(ab[s]), "us": round(1e3 * ms, 2),
                   "achieved_gbs": round(gbs, 1), "frac": round(gbs / hbm, 4)}
     if "window_scores" in stage_ms and wl.dtype == "bf16":
-        flops = 2.0 * wl.hq * wl.window * wl.head_dim * float(2 * np.sum(n) - len(n) * wl.window)
-        tf = flops / (stage_ms["window_scores"] * 1e-3) / 1e12
-        peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
-        out["window_scores"]["tensor"] = {"flops": flops, "achieved_tflops": round(tf, 1),
-                                          "peak_tflops": peak, "frac": round(tf / peak, 4),
-                                          "peak_source": "measured sustained bf16 (MEASURED_PEAKS.json)"}
+        per_key = 2.0 * wl.hq * wl.window * wl.head_dim
+        method = per_key * float(np.sum(n))
+        executed = per_key * float(2 * np.sum(n) - len(n) * wl.window)
+        sec = stage_ms["window_scores"] * 1e-3
+        peak = float(peaks["bf16_tflops"])
+        out["window_scores"]["tensor"] = {
+            "flops": method, "achieved_tflops": round(method / sec / 1e12, 1), "peak_tflops": peak,
+            "frac": round(method / sec / 1e12 / peak, 4),
+            "flops_rule": "the method's contraction: 2 Hq W d flops per key, one pass over the N keys",
+            "executed_flops": executed, "executed_tflops": round(executed / sec / 1e12, 1),
+            "executed_frac": round(executed / sec / 1e12 / peak, 4),
+            "executed_rule": "two passes as the kernel runs them: N keys (row statistics) + N - W keys (sums)",
+            "peak_source": "measured burst bf16 (MEASURED_PEAKS.json bf16_tflops): the stage is timed alone"}
     return out
 
 
@@ -242,33 +265,43 @@ def profiled_traffic(stage, workload):
 # our arm
 # ---------------------------------------------------------------------------
 
-def run_ours(args, wl, alpha, world, rank, local, dist):
-    import torch
-    from paper_2512_21859_gb300 import binding as tb
+STAGES = ["decode_attn", "window_scores", "select_topk", "gather_kv"]
 
-    torch.cuda.set_device(local)
-    tb.load()
-    dev = torch.device("cuda", local)
-    stream = torch.cuda.current_stream(dev)
-    lay = inputs.make_layer(wl, rank, alpha=alpha)
-    n, a = lay["n"], lay["alpha"]
-    B = len(n)
-    ab = alg_bytes(wl, n, a, [r + 1 for r in [retained(nb, wl.window, x)[1] for nb, x in zip(n, a)]])
-    R = ab["R"]
-    lens_h = [r + 1 for r in R]
-    e = elem_bytes(wl)
-    layer_bytes = 2 * wl.hkv * int(np.sum(n)) * wl.head_dim * e
+
+def to_device(torch, wl, x, dev):
+    if wl.dtype == "bf16":
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
+    return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+
+def load_workload(torch, wl, rank, dev):
+    """One layer's eviction inputs on the device, cloned into enough
+    rotating buffers that their K and V together exceed L2 three times
+    over. The inputs do not depend on alpha (it only sets the budget)."""
+    lay = inputs.make_layer(wl, rank)
+    n = lay["n"]
+    layer_bytes = 2 * wl.hkv * int(np.sum(n)) * wl.head_dim * elem_bytes(wl)
     L = int(min(64, max(2, math.ceil(3 * L2_BYTES / layer_bytes))))
+    base = {k: to_device(torch, wl, lay[k], dev) for k in ("q_win", "K", "V")}
+    layers = [{k: (v if li == 0 else v.clone()) for k, v in base.items()} for li in range(L)]
+    return {"wl": wl, "lay": lay, "n": n, "L": L, "layer_bytes": layer_bytes, "layers": layers}
 
-    def to_dev(x):
-        if wl.dtype == "bf16":
-            return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
-        return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
 
+def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
+    """Descriptors and per-buffer outputs of one eviction ratio; runs every
+    stage once per buffer (filling each compacted cache) and checks the
+    status words. The decode stage gets its own rotation of compacted caches
+    (copies of the buffers' own) large enough that one replay of its graph
+    reads more than three times L2."""
+    wl, n, lay = W["wl"], W["n"], W["lay"]
+    B = len(n)
+    R = [retained(nb, wl.window, x)[1] for nb, x in zip(n, alpha_vec)]
+    lens_h = [r + 1 for r in R]
+    ab = alg_bytes(wl, n, alpha_vec, lens_h)
     desc = tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, window=wl.window,
                         pool_k=wl.pool_k, dtype=tb.TB_BF16 if wl.dtype == "bf16" else tb.TB_F32,
-                        n=n, alpha=a, kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)),
-                        out_cap=[r + 1 for r in R])
+                        n=n, alpha=alpha_vec, kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)),
+                        out_cap=lens_h)
     score_rows, idx_rows = tb.tb_evict_layout(desc)
     ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
                           cache_offset=desc.out_offset, cache_cap=desc.out_cap,
@@ -276,14 +309,12 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     ews = tb.tb_evict_workspace_size(desc)
     dws = tb.tb_decode_workspace_size(ddesc)
     step_in = inputs.make_decode_step(wl, rank, 1, B)
-
-    base = {k: to_dev(lay[k]) for k in ("q_win", "K", "V")}
-    q_dec = to_dev(step_in["q"])
-    kn, vn = to_dev(step_in["k_new"]), to_dev(step_in["v_new"])
-    layers = []
-    for li in range(L):
-        d = {k: (v if li == 0 else v.clone()) for k, v in base.items()}
-        d["Kc"] = torch.zeros((wl.hkv, desc.out_rows, wl.head_dim), dtype=base["K"].dtype, device=dev)
+    q_dec = to_device(torch, wl, step_in["q"], dev)
+    kn, vn = to_device(torch, wl, step_in["k_new"], dev), to_device(torch, wl, step_in["v_new"], dev)
+    bufs = []
+    for lb in W["layers"]:
+        d = dict(lb)
+        d["Kc"] = torch.zeros((wl.hkv, desc.out_rows, wl.head_dim), dtype=lb["K"].dtype, device=dev)
         d["Vc"] = torch.zeros_like(d["Kc"])
         for b in range(B):   # the decode token's own K/V row, after the retained rows
             row = int(desc.out_offset[b]) + R[b]
@@ -295,10 +326,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         d["dws"] = torch.empty(dws, dtype=torch.uint8, device=dev)
         tb.tb_decode_workspace_prepare(ddesc, d["dws"], stream=stream)
         d["out"] = torch.empty((B, wl.hq, wl.head_dim), dtype=torch.float32, device=dev)
-        layers.append(d)
+        bufs.append(d)
     lens = torch.tensor(lens_h, dtype=torch.int32, device=dev)
-
-    stages = ["decode_attn", "window_scores", "select_topk", "gather_kv"]
 
     def stage_call(name, d, st):
         if name == "decode_attn":
@@ -310,15 +339,80 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         else:
             tb.tb_gather_kv(desc, d["idx"], d["K"], d["V"], d["Kc"], d["Vc"], stream=st)
 
-    # eager once per buffer (fills every compacted cache), then capture each
-    # layer's step, and each stage alone, into CUDA graphs
-    for d in layers:
-        for name in stages:
+    for d in bufs:
+        for name in STAGES:
             stage_call(name, d, stream)
     torch.cuda.synchronize(dev)
-    for d in layers:
+    for d in bufs:
         st, raw = tb.tb_read_status(d["ews"], stream=stream)
         assert st == tb.TB_OK, raw
+    # the decode's own rotation: each extra buffer a copy of a compacted cache
+    # the eviction wrote, with its own prepared workspace
+    Ld = int(min(64, max(len(bufs), math.ceil(3 * L2_BYTES / ab["decode_attn"]))))
+    dec_bufs = list(bufs)
+    for i in range(len(bufs), Ld):
+        src = bufs[i % len(bufs)]
+        d = {"Kc": src["Kc"].clone(), "Vc": src["Vc"].clone(),
+             "dws": torch.empty(dws, dtype=torch.uint8, device=dev), "out": torch.empty_like(src["out"])}
+        tb.tb_decode_workspace_prepare(ddesc, d["dws"], stream=stream)
+        dec_bufs.append(d)
+    torch.cuda.synchronize(dev)
+    return {"desc": desc, "ddesc": ddesc, "bufs": bufs, "dec_bufs": dec_bufs, "R": R, "ab": ab,
+            "stage_call": stage_call, "step_in": step_in, "ews": ews, "dws": dws}
+
+
+def check_decode_status(tb, stream, S):
+    for d in S["dec_bufs"]:
+        st, raw = tb.tb_read_status(d["dws"], stream=stream)
+        assert st == tb.TB_OK, raw
+
+
+def sweep_points(torch, tb, W, alphas, rank, dev, stream, peaks, steps):
+    """The metric's alpha axis: per-stage device time per layer (each stage
+    timed as in the headline) and the eviction and decode HBM fractions at
+    each alpha, on the same rotated inputs."""
+    wl = W["wl"]
+    hbm = float(peaks["hbm_gbs"])
+    cap = torch.cuda.Stream(dev)
+    rows = []
+    for alpha in alphas:
+        avec = np.full(len(W["n"]), float(alpha))
+        S = setup_alpha(torch, tb, W, avec, rank, dev, stream)
+        ms, _ = time_stages(torch, dev, stream, cap, S, steps)
+        check_decode_status(tb, stream, S)
+        ab = S["ab"]
+        ev_ms = ms["window_scores"] + ms["select_topk"] + ms["gather_kv"]
+        ev_gbs = ab["evict"] / (ev_ms * 1e-3) / 1e9
+        dec_gbs = ab["decode_attn"] / (ms["decode_attn"] * 1e-3) / 1e9
+        rows.append({"workload": wl.name, "alpha": float(alpha), "R": int(S["R"][0]),
+                     "us": {s: round(1e3 * v, 2) for s, v in ms.items()},
+                     "evict_us": round(1e3 * ev_ms, 2), "evict_gbs": round(ev_gbs, 1),
+                     "evict_frac": round(ev_gbs / hbm, 4), "decode_gbs": round(dec_gbs, 1),
+                     "decode_frac": round(dec_gbs / hbm, 4),
+                     "decode_rotation": len(S["dec_bufs"])})
+        del S
+        torch.cuda.empty_cache()
+    return rows
+
+
+def run_ours(args, wl, alpha, world, rank, local, dist):
+    import torch
+    from paper_2512_21859_gb300 import binding as tb
+
+    torch.cuda.set_device(local)
+    tb.load()
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    W = load_workload(torch, wl, rank, dev)
+    n = W["n"]
+    a = inputs.request_shapes(wl, alpha)[1]
+    L = W["L"]
+    S = setup_alpha(torch, tb, W, a, rank, dev, stream)
+    ab, R, desc, ddesc = S["ab"], S["R"], S["desc"], S["ddesc"]
+    stage_call = S["stage_call"]
+    layers = S["bufs"]
+
+    # each layer buffer's step (decode, then the eviction) captured into a CUDA graph
     cap = torch.cuda.Stream(dev)
     step_graphs = []
     kernels_per_step = None
@@ -326,7 +420,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         g = torch.cuda.CUDAGraph()
         c0 = tb.tb_launch_counter()
         with torch.cuda.graph(g, stream=cap):
-            for name in stages:
+            for name in STAGES:
                 stage_call(name, d, cap)
         kernels_per_step = tb.tb_launch_counter() - c0
         step_graphs.append(g)
@@ -353,42 +447,50 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     if dist:
         dist.barrier()
     total_ms = t0.elapsed_time(t1)
-    stage_ms, stage_timing = time_stages(torch, dev, stream, cap, layers, stages, stage_call, K)
+    stage_ms, stage_timing = time_stages(torch, dev, stream, cap, S, K)
     clocks = sampler.stop()
     launches = kernels_per_step * K
     total_ms = max_over_ranks(dist, total_ms, dev)
-    for d in layers:
-        st, raw = tb.tb_read_status(d["dws"], stream=stream)
-        assert st == tb.TB_OK, raw
+    check_decode_status(tb, stream, S)
     ms_step = total_ms / K
     value = job_value(world, ab["step"], K, total_ms)
 
-    # roofline of the dominant stage
+    # roofline of the dominant stage: algorithmic HBM bytes per launch over
+    # its per-launch time, against the measured copy bandwidth
     with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
         peaks = json.load(f)
     peak = float(peaks["hbm_gbs"])
-    dom = max(stages, key=lambda s: stage_ms[s])
+    dom = max(STAGES, key=lambda s: stage_ms[s])
     achieved = ab[dom] / (stage_ms[dom] * 1e-3) / 1e9
-    roof = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
-            "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
-            "traffic": profiled_traffic(dom, wl.name),
-            "alg_bytes_per_launch": ab[dom], "avg_launch_ms": round(stage_ms[dom], 5)}
     sroof = stage_rooflines(wl, n, ab, stage_ms, peaks)
+    roof = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+            "unit": "GB/s", "frac": round(achieved / peak, 4),
+            "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
+            "traffic": profiled_traffic(dom, wl.name),
+            "alg_bytes_per_launch": int(ab[dom]), "avg_launch_ms": round(stage_ms[dom], 5),
+            "bytes_rule": SURVEY_BYTES_RULE.get(dom, "")}
     if "tensor" in sroof.get(dom, {}):
-        # the window scoring is a dense bf16 contraction (two QK^T passes over
-        # the window rows: statistics, then normalised sums), so its roofline
-        # is the tensor rate; its HBM fraction stays in the stage table
-        t = sroof[dom]["tensor"]
-        roof.update({"bound": "tensor", "achieved": t["achieved_tflops"], "peak": t["peak_tflops"],
-                     "unit": "TFLOP/s", "frac": t["frac"],
-                     "peak_source": "measured sustained bf16 (MEASURED_PEAKS.json bf16_tflops_sustained)",
-                     "alg_flops_per_launch": t["flops"],
-                     "flops_rule": "2 Hq W d flops per key and pass: N keys (statistics) + N - W keys (sums)", "hbm_frac": sroof[dom]["frac"]})
+        roof["tensor"] = sroof[dom]["tensor"]
 
-    lse_var = None if args.no_variants else time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers,
+    lse_var = None if args.no_variants else time_lse_variant(torch, tb, dev, stream, wl, W["lay"], desc, layers,
                                                              stage_ms, ms_step, n, peaks)
 
-    e2e = run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R)
+    e2e = run_e2e(args, wl, tb, torch, dev, stream, W["lay"], desc, ddesc, S["ews"], S["dws"], S["step_in"],
+                  ab, R)
+
+    sweep = None
+    if not args.no_alpha_sweep:
+        del S, layers, step_graphs, stage_call
+        torch.cuda.empty_cache()
+        sweep = {"timing": "per stage as in stage_timing; each alpha on the same rotated inputs",
+                 "points": []}
+        for wname, alphas in ALPHA_SWEEP:
+            Wx = W if wname == wl.name else load_workload(torch, inputs.WORKLOADS[wname], rank, dev)
+            sweep["points"] += sweep_points(torch, tb, Wx, alphas, rank, dev, stream, peaks,
+                                            args.sweep_steps)
+            if Wx is not W:
+                del Wx
+                torch.cuda.empty_cache()
 
     evict_us = 1e3 * (stage_ms["window_scores"] + stage_ms["select_topk"] + stage_ms["gather_kv"])
     res = {
@@ -398,7 +500,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         "dtype": wl.dtype, "data": "synthetic (seeded Gaussian q/K/V with planted heavy hitters)",
         "config": {
             "workload": describe(wl, n, a), "alpha": float(a[0]) if len(set(a.tolist())) == 1 else a.tolist(),
-            "layers_rotated": L, "l2": "inputs larger than L2: %d rotating layer buffers of %.0f MB" % (L, layer_bytes / 1e6),
+            "layers_rotated": L, "l2": "inputs larger than L2: %d rotating layer buffers of %.0f MB" % (
+                L, W["layer_bytes"] / 1e6),
             "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
             "decode_call": "tb_decode_attn_prepared (workspace prepared once; no per-call clearing kernel)",
             "launch": "each step is one CUDA-graph replay of the four C-ABI calls",
@@ -409,9 +512,13 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                          "stages": {s: round(1e3 * v, 2) for s, v in stage_ms.items()}},
         "gbs": {"evict": round(ab["evict"] / (evict_us * 1e-6) / 1e9, 1),
                 "decode": round(ab["decode_attn"] / (stage_ms["decode_attn"] * 1e-3) / 1e9, 1)},
+        "frac_of_measured_hbm": {"evict": round(ab["evict"] / (evict_us * 1e-6) / 1e9 / peak, 4),
+                                 "decode": round(ab["decode_attn"] / (stage_ms["decode_attn"] * 1e-3) / 1e9 / peak, 4),
+                                 "step": round(value / world / peak, 4)},
         "frac_of_8tbs": round(value / world / NOMINAL_HBM_GBS, 4),
         "roofline": roof,
         "stage_roofline": sroof,
+        "alpha_sweep": sweep,
         "prefill_lse_variant": lse_var,
         "e2e": e2e,
         "gpu_launches": int(launches),
@@ -484,7 +591,7 @@ def time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, st
     us = 1e3 * t0.elapsed_time(t1) / (reps * len(layers))
     flops = 2.0 * wl.hq * wl.window * wl.head_dim * float(np.sum(n) - len(n) * wl.window)
     tf = flops / (us * 1e-6) / 1e12
-    peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+    peak = float(peaks["bf16_tflops"])
     # the step with this call in place of tb_window_scores: the measured step
     # time less the difference of the two calls' stage times
     step = 1e3 * (step_ms - stage_ms["window_scores"]) + us
@@ -495,22 +602,24 @@ def time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, st
             "note": "one QK^T pass over the prefix keys; the window rows' log-sum-exp comes from the prefill"}
 
 
-def time_stages(torch, dev, stream, cap, layers, stages, stage_call, K):
+def time_stages(torch, dev, stream, cap, S, K):
     """Per-stage device time per launch: for each stage one CUDA graph of
-    that stage's call on every rotated layer buffer in turn (inputs larger
-    than L2 across the rotation), replayed with CUDA events around the
-    replays. This is the stage's launch duration plus the gap between two
-    kernels of a graph; the step graph's own time (the headline) also holds
-    the interaction between stages (e.g. the L2 write-back of the gather's
-    output while the next decode reads)."""
-    L = len(layers)
-    reps = max(3, -(-K // L))
-    out = {}
-    for name in stages:
+    that stage's call on every buffer of its rotation in turn (the eviction
+    stages over the layer buffers, whose K and V exceed L2 three times; the
+    decode over its own rotation of compacted caches, likewise beyond L2),
+    replayed with CUDA events around the replays. This is the stage's
+    launch duration plus the gap between two kernels of a graph; the step
+    graph's own time (the headline) also holds the interaction between
+    stages (e.g. the L2 write-back of the gather's output)."""
+    out, rot = {}, {}
+    for name in STAGES:
+        bufs = S["dec_bufs"] if name == "decode_attn" else S["bufs"]
+        L = len(bufs)
+        reps = max(3, -(-K // L))
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=cap):
-            for d in layers:
-                stage_call(name, d, cap)
+            for d in bufs:
+                S["stage_call"](name, d, cap)
         with torch.cuda.stream(stream):
             for _ in range(2):
                 g.replay()
@@ -524,17 +633,26 @@ def time_stages(torch, dev, stream, cap, layers, stages, stage_call, K):
             t1.record(stream)
         torch.cuda.synchronize(dev)
         out[name] = t0.elapsed_time(t1) / (reps * L)
-    return out, ("per stage: one CUDA graph of the stage's call on each of the %d rotated layer "
-                 "buffers, %d replays between CUDA events" % (L, reps))
+        rot[name] = L
+        del g
+    return out, ("per stage: one CUDA graph of the stage's call on each buffer of its rotation "
+                 "(%d layer buffers; the decode over %d compacted caches), replayed between CUDA events"
+                 % (rot["window_scores"], rot["decode_attn"]))
 
 
 def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_in, ab, R):
     """The same step through the public API from pinned HOST buffers: every
-    step copies its inputs host->device and reads its results back."""
+    step copies its inputs host->device and reads its results back. With one
+    request the copies are issued per KV head on a copy stream and each
+    head's eviction (tb_score_evict on that head's rows) starts once its
+    rows have landed, so the evictions overlap the remaining copies; the
+    decode follows the last head. The serial form (all copies, then the
+    whole eviction) and a copy-only step are timed beside it."""
     steps = args.e2e_steps if args.e2e_steps is not None else min(args.steps, 10)
     if steps <= 0:
         return None
     B = len(lay["n"])
+    G = wl.group
 
     def host(x):
         if wl.dtype == "bf16":
@@ -559,38 +677,91 @@ def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_i
     idx_h = torch.empty(idx.shape, dtype=torch.int32).pin_memory()
     out_h = torch.empty(out.shape, dtype=torch.float32).pin_memory()
     rows = [int(desc.out_offset[b]) + R[b] for b in range(B)]
+    copy_stream = torch.cuda.Stream(dev)
+    per_head = B == 1
+    if per_head:   # one KV head's eviction: its G query heads, its K and V rows
+        hdesc = tb.EvictDesc(hq=G, hkv=1, head_dim=wl.head_dim, window=wl.window, pool_k=wl.pool_k,
+                             dtype=desc.dtype, n=desc.n, alpha=desc.alpha, kv_offset=desc.kv_offset,
+                             kv_rows=desc.kv_rows, out_offset=desc.out_offset, out_cap=desc.out_cap,
+                             out_rows=desc.out_rows, flags=desc.flags)
+        hws = torch.empty(tb.tb_evict_workspace_size(hdesc), dtype=torch.uint8, device=dev)
+        landed = [torch.cuda.Event() for _ in range(wl.hkv)]
 
-    def one():
+    def tail():
+        qd.copy_(hq, non_blocking=True)
+        kd.copy_(hk, non_blocking=True)
+        vd.copy_(hv, non_blocking=True)
+        for b in range(B):
+            Kc[:, rows[b]] = kd[:, b]
+            Vc[:, rows[b]] = vd[:, b]
+        tb.tb_decode_attn_prepared(ddesc, qd, Kc, Vc, lens, out, dw, stream=stream)
+        idx_h.copy_(idx, non_blocking=True)
+        out_h.copy_(out, non_blocking=True)
+
+    def serial():
+        with torch.cuda.stream(stream):
+            for k in d:
+                d[k].copy_(h[k], non_blocking=True)
+            tb.tb_score_evict(desc, d["q_win"], d["K"], d["V"], idx, Kc, Vc, None, ew, stream=stream)
+            tail()
+
+    def overlapped():
+        copy_stream.wait_stream(stream)
+        with torch.cuda.stream(copy_stream):
+            d["q_win"].copy_(h["q_win"], non_blocking=True)
+            for g in range(wl.hkv):
+                d["K"][g].copy_(h["K"][g], non_blocking=True)
+                d["V"][g].copy_(h["V"][g], non_blocking=True)
+                landed[g].record(copy_stream)
+        with torch.cuda.stream(stream):
+            for g in range(wl.hkv):
+                stream.wait_event(landed[g])
+                tb.tb_score_evict(hdesc, d["q_win"][:, g * G:(g + 1) * G], d["K"][g], d["V"][g], idx[g], Kc[g],
+                                  Vc[g], None, hws, stream=stream)
+            tail()
+
+    def copy_only():
         with torch.cuda.stream(stream):
             for k in d:
                 d[k].copy_(h[k], non_blocking=True)
             qd.copy_(hq, non_blocking=True)
             kd.copy_(hk, non_blocking=True)
             vd.copy_(hv, non_blocking=True)
-            tb.tb_score_evict(desc, d["q_win"], d["K"], d["V"], idx, Kc, Vc, None, ew, stream=stream)
-            for b in range(B):
-                Kc[:, rows[b]] = kd[:, b]
-                Vc[:, rows[b]] = vd[:, b]
-            tb.tb_decode_attn_prepared(ddesc, qd, Kc, Vc, lens, out, dw, stream=stream)
-            idx_h.copy_(idx, non_blocking=True)
-            out_h.copy_(out, non_blocking=True)
 
-    for _ in range(2):
-        one()
-    torch.cuda.synchronize(dev)
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    t0.record(stream)
-    for _ in range(steps):
-        one()
-    t1.record(stream)
-    torch.cuda.synchronize(dev)
-    ms = t0.elapsed_time(t1) / steps
+    def timed(fn):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize(dev)
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(steps):
+            fn()
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+        return t0.elapsed_time(t1) / steps
+
+    ms_serial = timed(serial)
+    idx_serial = idx_h.clone()
+    ms, same_idx = ms_serial, None
+    if per_head:
+        ms = timed(overlapped)
+        st, raw = tb.tb_read_status(hws, stream=stream)
+        assert st == tb.TB_OK, raw
+        same_idx = bool(torch.equal(idx_h, idx_serial))
+    ms_copy = timed(copy_only)
     h2d = sum(v.numel() * v.element_size() for v in h.values()) + sum(
         v.numel() * v.element_size() for v in (hq, hk, hv))
     d2h = idx_h.numel() * 4 + out_h.numel() * 4
     return {"value": round(ab["step"] / (ms * 1e-3) / 1e9, 1), "unit": "GB/s", "ms_per_step": round(ms, 4),
-            "steps": steps, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+            "steps": steps, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "form": ("per-KV-head copies on a copy stream, each head's tb_score_evict after its rows land"
+                     if per_head else "all copies, then tb_score_evict and the decode"),
+            "serial_ms_per_step": round(ms_serial, 4),
+            "copy_only_ms_per_step": round(ms_copy, 4),
+            "pinned_h2d_gbs": round(h2d / (ms_copy * 1e-3) / 1e9, 1),
+            "copy_bound_frac": round(ms_copy / ms, 4),
+            "per_head_idx_equal_batched": same_idx}
 
 
 def describe(wl, n, a):
@@ -830,6 +1001,8 @@ def main(argv=None):
         return 0
     dist = dist_init(world, True)
     alphas = [float(x) for x in args.sweep.split(",")] if args.sweep else [args.alpha]
+    if args.sweep:   # one line per alpha already: no per-alpha table inside each
+        args.no_alpha_sweep = True
     base_cpu = None
     for alpha in alphas:
         res = run_ours(args, wl, alpha, world, rank, local, dist)

@@ -286,12 +286,25 @@ tb_status tb_read_status(const void *workspace, size_t workspace_bytes,
                          tb_stream_t stream, int32_t *raw);
 
 /*
- * Diagnostic: y[i] = 2^x[i] computed by the FMA-pipe exponential the scoring
- * kernels use for part of their softmax terms (Cody-Waite range reduction and
- * a degree-5 polynomial; relative error below 2.2e-7 for x in [-125, 0.5];
- * inputs below -125 are clamped there). x, y: device float arrays of n.
+ * Diagnostic of the bounded device-side waits behind TB_ERR_TIMEOUT
+ * (failure detection; the paper has no counterpart). Every kernel here
+ * waits on its barriers with a time limit and, when it runs out, raises the
+ * workspace status word, waits for its own copies in flight, frees its
+ * tensor memory and returns instead of hanging. This call runs that exit on
+ * purpose: one CTA starts a 4 KB copy into shared memory, then waits on a
+ * barrier that nothing completes (arrive = 0) for limit_ns nanoseconds of
+ * the GPU timer, or on one it completes itself first (arrive = 1).
+ *  - workspace: device, 256-byte aligned, at least 256 + 4096 bytes; its
+ *    status word is cleared first, the 4 KB after the first 256 bytes are
+ *    read (any contents). Afterwards tb_read_status on it gives
+ *    TB_ERR_TIMEOUT (arrive = 0) or TB_OK (arrive = 1).
+ *  - limit_ns: 10,000 .. 1,000,000,000 (10 us .. 1 s).
+ * Errors: TB_ERR_WORKSPACE (missing, small or misaligned workspace),
+ * TB_ERR_INVALID_ARG (limit out of range, arrive not 0 or 1), TB_ERR_CUDA.
  */
-tb_status tb_diag_exp2(const float *x, float *y, int64_t n, tb_stream_t stream);
+tb_status tb_diag_bounded_wait(void *workspace, size_t workspace_bytes,
+                               uint64_t limit_ns, int32_t arrive,
+                               tb_stream_t stream);
 
 /* Size of the device array tb_decode_attn_noalloc uses as its scratch. */
 #define TB_NOALLOC_SCRATCH_BYTES (4u << 20)
@@ -308,19 +321,34 @@ tb_status tb_diag_exp2(const float *x, float *y, int64_t n, tb_stream_t stream);
  * library holds until the process exits. It allocates nothing.
  *  - A descriptor whose tb_decode_workspace_size exceeds the array returns
  *    TB_ERR_WORKSPACE before any launch; use tb_decode_attn instead.
- *  - It runs on the calling thread's current device. The first call on each
- *    device looks up the array's device address there (cudaGetSymbolAddress)
- *    and keeps it, so make that first call before any stream capture.
+ *  - It runs on the calling thread's current device. The first call in each
+ *    CUDA context (per device; a context made after cudaDeviceReset, or a
+ *    driver-API context of the caller's, counts as new) looks up the array's
+ *    device address there (cudaGetSymbolAddress) and keeps it, so make that
+ *    first call before any stream capture.
  *  - Every call on a device shares the one array, which keeps the previous
  *    call's contents: calls that overlap on the GPU (other streams, other
- *    threads) race and must be serialised by the caller.
- *  - A length above its cap is clamped as in tb_decode_attn, but the range
- *    flag cannot be read back (there is no caller workspace to read).
+ *    threads) race and must be serialised by the caller. Each call clears
+ *    the array's status word and split counters before its kernels run.
+ *  - A length above its cap is clamped and flagged as in tb_decode_attn,
+ *    and a bounded wait that gives up raises the timeout flag (the output
+ *    is then not valid); both flags land in the array's status word, which
+ *    tb_decode_noalloc_status reads back.
  */
 tb_status tb_decode_attn_noalloc(const tb_decode_desc *desc, const void *q,
                                  const void *Kc, const void *Vc,
                                  const int32_t *lens, void *out,
                                  tb_stream_t stream);
+
+/*
+ * Status word of the array tb_decode_attn_noalloc uses, on the current
+ * device: waits for `stream` (the stream of the calls to check), then reports
+ * what the last tb_decode_attn_noalloc call on this device raised, as
+ * tb_read_status does: TB_OK, TB_ERR_TIMEOUT or TB_ERR_INVALID_ARG (a length
+ * above its cap). *raw (if not NULL) receives the word. Allocates nothing.
+ * Errors: TB_ERR_CUDA if the synchronisation or the read fails.
+ */
+tb_status tb_decode_noalloc_status(tb_stream_t stream, int32_t *raw);
 
 /*
  * Execution-time model of "Profiling-based Fitting" (Eq. 6a and 6b), in

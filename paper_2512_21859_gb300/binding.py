@@ -24,7 +24,7 @@ __all__ = [
     "TB_EVICT_AVG_POOL", "tb_evict_layout", "tb_evict_workspace_size",
     "tb_window_scores", "tb_window_scores_lse", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
-    "tb_decode_attn_noalloc", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_exp2",
+    "tb_decode_attn_noalloc", "tb_decode_noalloc_status", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_bounded_wait",
     "tb_decode_workspace_prepare", "tb_decode_attn_prepared",
     "TimeModel", "tb_wcet", "tb_alpha_star", "tb_fit_time_model",
 ]
@@ -108,9 +108,10 @@ def load():
         "tb_decode_attn": (I, [P, P, P, P, P, P, P, SZ, P]),
         "tb_read_status": (I, [P, SZ, P, ctypes.POINTER(I)]),
         "tb_decode_attn_noalloc": (I, [P, P, P, P, P, P, P]),
+        "tb_decode_noalloc_status": (I, [P, ctypes.POINTER(I)]),
         "tb_decode_workspace_prepare": (I, [P, P, SZ, P]),
         "tb_decode_attn_prepared": (I, [P, P, P, P, P, P, P, SZ, P]),
-        "tb_diag_exp2": (I, [P, P, ctypes.c_int64, P]),
+        "tb_diag_bounded_wait": (I, [P, SZ, ctypes.c_uint64, I, P]),
         "tb_wcet": (I, [P, ctypes.c_int64, ctypes.c_double, ctypes.c_int64, ctypes.POINTER(ctypes.c_double)]),
         "tb_alpha_star": (I, [P, ctypes.c_int64, ctypes.c_double, ctypes.c_double, ctypes.c_int64,
                               ctypes.c_double, ctypes.c_double, ctypes.c_double,
@@ -358,9 +359,23 @@ def tb_decode_attn_noalloc(desc: DecodeDesc, q, Kc, Vc, lens, out, stream=None):
                                          _stream(stream)), "tb_decode_attn_noalloc")
 
 
-def tb_diag_exp2(x, y, stream=None):
-    """y = 2^x by the scoring kernels' FMA-pipe exponential (diagnostic)."""
-    _check(load().tb_diag_exp2(_ptr(x), _ptr(y), int(x.numel()), _stream(stream)), "tb_diag_exp2")
+def tb_decode_noalloc_status(stream=None):
+    """(status, raw word) of the array tb_decode_attn_noalloc uses on the
+    current device, after waiting for the stream."""
+    raw = ctypes.c_int32()
+    st = load().tb_decode_noalloc_status(_stream(stream), ctypes.byref(raw))
+    if st not in (TB_OK, TB_ERR_TIMEOUT, TB_ERR_INVALID_ARG):
+        raise TbError(st, "tb_decode_noalloc_status")
+    return st, raw.value
+
+
+def tb_diag_bounded_wait(workspace, limit_ns: int, arrive: int = 0, workspace_bytes=None, stream=None):
+    """Runs the bounded-wait exit on purpose (diagnostic): a wait on a barrier
+    that nothing completes gives up after limit_ns; tb_read_status on the
+    workspace then reports TB_ERR_TIMEOUT (TB_OK with arrive=1)."""
+    w, wb = _ws(workspace, workspace_bytes)
+    _check(load().tb_diag_bounded_wait(w, wb, int(limit_ns), int(arrive), _stream(stream)),
+           "tb_diag_bounded_wait")
 
 
 def tb_read_status(workspace, workspace_bytes=None, stream=None):

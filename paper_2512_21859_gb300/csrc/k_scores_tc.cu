@@ -53,12 +53,6 @@ constexpr int kProducerWarp = 16;  // TMA issue; also owns the TMEM allocation
 constexpr int kMmaWarp = 17;       // tcgen05.mma issue
 constexpr uint32_t kTmemCols = 512;
 constexpr int kBoxBytes = 128 * 128;  // one TMA box: 128 rows x 64 bf16
-// Of every 32 exponentials an epilogue thread takes, the first kMufuElems go
-// to the MUFU unit and the rest to the FMA pipes (tc::exp2_poly2). Measured on
-// GB300: sending 4 or 8 of 32 to the FMA pipes slowed both passes (they are
-// bound by streaming K, and the epilogue by latency, not by MUFU throughput),
-// so all of them use MUFU.
-constexpr int kMufuElems = 32;
 // Set in the grid-barrier word when a row maximum is too large for the fp64
 // row sums (those heads then merge their partials the slow way).
 constexpr uint32_t kSumOverflowBit = 0x80000000u;
@@ -213,16 +207,8 @@ __device__ __forceinline__ float vote_sum(const float (&v)[64], float c, const f
     const float4 nc = *reinterpret_cast<const float4*>(bias + i);
     const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), c2, tc::pk2(nc.x, nc.y)));
     const float2 y = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), c2, tc::pk2(nc.z, nc.w)));
-    float2 ex, ey;
-    if ((i & 31) < kMufuElems) {
-      ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
-      ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
-    } else {
-      ex = tc::exp2_poly2(x.x, x.y);
-      ey = tc::exp2_poly2(y.x, y.y);
-    }
-    a0 = tc::add2(a0, tc::pk2(ex.x, ex.y));
-    a1 = tc::add2(a1, tc::pk2(ey.x, ey.y));
+    a0 = tc::add2(a0, tc::pk2(fast_exp2(x.x), fast_exp2(x.y)));
+    a1 = tc::add2(a1, tc::pk2(fast_exp2(y.x), fast_exp2(y.y)));
   }
   const float2 s01 = tc::upk2(tc::add2(a0, a1));
   return s01.x + s01.y;
@@ -452,16 +438,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 64; i += 4) {
               const float2 x = tc::upk2(tc::fma2(tc::pk2(v[i], v[i + 1]), cc, mm));
               const float2 y = tc::upk2(tc::fma2(tc::pk2(v[i + 2], v[i + 3]), cc, mm));
-              float2 ex, ey;
-              if ((i & 31) < kMufuElems) {
-                ex = make_float2(fast_exp2(x.x), fast_exp2(x.y));
-                ey = make_float2(fast_exp2(y.x), fast_exp2(y.y));
-              } else {
-                ex = tc::exp2_poly2(x.x, x.y);
-                ey = tc::exp2_poly2(y.x, y.y);
-              }
-              acc0 = tc::add2(acc0, tc::pk2(ex.x, ex.y));
-              acc1 = tc::add2(acc1, tc::pk2(ey.x, ey.y));
+              acc0 = tc::add2(acc0, tc::pk2(fast_exp2(x.x), fast_exp2(x.y)));
+              acc1 = tc::add2(acc1, tc::pk2(fast_exp2(y.x), fast_exp2(y.y)));
             }
             const float2 s01 = tc::upk2(tc::add2(acc0, acc1));
             const float term = (s01.x + s01.y) - l_comp;

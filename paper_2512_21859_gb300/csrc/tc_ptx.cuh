@@ -2,9 +2,10 @@
 // loads, tcgen05 (TMEM allocation, MMA, commit, loads, fences) and the shared
 // memory / instruction descriptors of tcgen05.mma.kind::f16.
 //
-// Every wait here is bounded: after kWaitNs nanoseconds of %globaltimer it
-// raises the CTA's abort flag and the device status word and returns false,
-// so a kernel that loses a barrier arrival ends instead of hanging the GPU.
+// Every wait here is bounded: after kWaitNs nanoseconds of %globaltimer (or
+// the limit the caller passes) it raises the CTA's abort flag and the device
+// status word and returns false, so a kernel that loses a barrier arrival
+// ends instead of hanging the GPU.
 #pragma once
 
 #include <cuda.h>
@@ -61,16 +62,17 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for the phase of parity `parity` to complete. Returns false (and
-// raises *abort and the status word) on timeout, or if another warp aborted.
+// raises *abort and the status word) after limit_ns of waiting, or if
+// another warp aborted.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          int32_t* status) {
+                                          int32_t* status, uint64_t limit_ns = kWaitNs) {
   if (mbar_test(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t spin = 0;; ++spin) {
     if (mbar_test(bar, parity)) return true;
     if ((spin & 63u) == 63u) {
       if (*abort) return false;
-      if (globaltimer() - t0 > kWaitNs) {
+      if (globaltimer() - t0 > limit_ns) {
         *abort = 1;
         atomicOr(status, kStatusTimeout);
         return false;
@@ -93,6 +95,17 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_addr(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+      : "memory");
+}
+
+// Untiled bulk copy of `bytes` (a multiple of 16; both addresses 16-byte
+// aligned) from global to shared memory, completing on bar.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_addr(bar))
       : "memory");
 }
 
@@ -238,33 +251,6 @@ __device__ __forceinline__ uint64_t sub2(uint64_t a, uint64_t b) {
   uint64_t d;
   asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
-}
-
-// 2^x for a pair of x <= ~0.5 on the FMA pipes instead of the MUFU unit (about
-// 32 exponentials per SM per clock on GB300, as ncu's XU-pipe counts of the
-// scoring kernel put it). Cody-Waite split x = n + f with n
-// = round(x) (by adding 1.5 * 2^23) and f in [-0.5, 0.5]; 2^f by a degree-5
-// polynomial fitted for minimum relative error (exp2_poly_fit.py: 2.1e-7 in
-// fp32); 2^n added to the exponent field. x is clamped at -125 so that the
-// result stays a normal float; 2^-125 is far below anything that matters here.
-__device__ __forceinline__ float2 exp2_poly2(float x0, float x1) {
-  x0 = fmaxf(x0, -125.f);
-  x1 = fmaxf(x1, -125.f);
-  const uint64_t x = pk2(x0, x1);
-  const uint64_t magic = pk2(12582912.f, 12582912.f);  // 1.5 * 2^23
-  const uint64_t r = add2(x, magic);
-  const uint64_t f = sub2(x, sub2(r, magic));
-  uint64_t p = fma2(pk2(1.327647245e-03f, 1.327647245e-03f), f,
-                    pk2(9.675540961e-03f, 9.675540961e-03f));
-  p = fma2(p, f, pk2(5.550713092e-02f, 5.550713092e-02f));
-  p = fma2(p, f, pk2(2.402212024e-01f, 2.402212024e-01f));
-  p = fma2(p, f, pk2(6.931469440e-01f, 6.931469440e-01f));
-  p = fma2(p, f, pk2(1.000000119e+00f, 1.000000119e+00f));
-  const float2 pf = upk2(p), rf = upk2(r);
-  // low bits of r hold n (+ the magic's zero low bits): n << 23 shifts them into
-  // the exponent field, the magic's own bits shift out
-  return make_float2(__uint_as_float(__float_as_uint(pf.x) + (__float_as_uint(rf.x) << 23)),
-                     __uint_as_float(__float_as_uint(pf.y) + (__float_as_uint(rf.y) << 23)));
 }
 
 __device__ __forceinline__ float max3(float a, float b, float c) {

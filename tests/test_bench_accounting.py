@@ -6,8 +6,9 @@ from the definitions, independently of bench.py's code:
       (K read once to score; retained K and V rows read and written),
   decode bytes   = 2 e Hkv d len + B Hq d (e + 4)
       (K and V of the compacted cache; the query and the fp32 output),
-  scoring flops  = 2 Hq W d (N + (N - W))
-      (two QK^T passes over the window rows: N keys, then the N - W prefix keys),
+  scoring flops  = 2 Hq W d N (the method's one Q K^T over the N keys),
+      executed as 2 Hq W d (N + (N - W)) by the two-pass kernel
+      (N keys for the row statistics, then the N - W prefix keys),
 with R = k + W and k = ceil((1 - alpha) N) prefix rows (Eq. 8 reading).
 """
 import os
@@ -56,10 +57,17 @@ def test_128k_alpha_point_nine():
     assert ab["decode_attn"] == 2 * 2 * 8 * 128 * 13173 + 32 * 128 * (2 + 4) == 53_981_184
     peaks = {"hbm_gbs": 6790.3, "bf16_tflops": 1904.5, "bf16_tflops_sustained": 1717.4}
     roof = bench.stage_rooflines(wl, n, ab, {"window_scores": 0.1, "decode_attn": 0.01}, peaks)
-    flops = 2 * 32 * 64 * 128 * (131072 + (131072 - 64))
-    assert roof["window_scores"]["tensor"]["flops"] == flops == 137_405_399_040
-    # 0.1 ms per launch: 1374.05 TFLOP/s against the sustained 1717.4
-    assert roof["window_scores"]["tensor"]["frac"] == pytest.approx(flops / 1e-4 / 1e12 / 1717.4, abs=1e-4)
+    method = 2 * 32 * 64 * 128 * 131072
+    executed = 2 * 32 * 64 * 128 * (131072 + (131072 - 64))
+    t = roof["window_scores"]["tensor"]
+    assert t["flops"] == method == 68_719_476_736
+    assert t["executed_flops"] == executed == 137_405_399_040
+    # 0.1 ms per launch: 687.19 TFLOP/s of the method's flops against the burst 1904.5
+    assert t["frac"] == pytest.approx(687.19476736 / 1904.5, abs=1e-4)
+    assert t["executed_frac"] == pytest.approx(1374.0539904 / 1904.5, abs=1e-4)
+    # the headline roofline is HBM: 268,959,744 bytes (K once + q_win) in 0.1 ms
+    assert ab["window_scores"] == 2 * 8 * 128 * 131072 + q_win == 268_959_744
+    assert roof["window_scores"]["frac"] == pytest.approx(2689.59744 / 6790.3, abs=1e-4)
     assert roof["decode_attn"]["achieved_gbs"] == pytest.approx(53_981_184 / 1e-5 / 1e9, rel=1e-3)
 
 

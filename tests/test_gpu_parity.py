@@ -72,19 +72,38 @@ def _check_evict(wl, lay, res, ref, heads=None):
     return excused
 
 
-def _decode_and_check(wl, lay, res, steps, heads_check=None, layer=0):
-    """Appends `steps` decode tokens one by one and checks every step."""
+def _decode_and_check(wl, lay, res, steps, heads_check=None, layer=0, check_at=None):
+    """Runs a decode loop of `steps` tokens after the eviction, the way a
+    caller's loop does: each step appends its own K/V row at lens[b] - 1
+    (Eq. 8's N_kv^i grows by one row per step) and describes the step with
+    max_len = the current longest length, so the split layout follows the
+    lengths as they grow. The step runs through tb_decode_attn_prepared on
+    one workspace prepared before the loop (the call the benchmark times).
+    At the steps in `check_at` (default: the first two, the middle and the
+    last; every step for short loops) the output is compared with the
+    oracle, and tb_decode_attn on the same inputs must give identical bits."""
     desc = res["desc"]
     B = desc.batch
     R = [request_slices(desc, b)[3] for b in range(B)]
     caps = [int(c) for c in desc.out_cap]
-    ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=DT[wl.dtype],
-                          cache_offset=desc.out_offset, cache_cap=caps, cache_rows=desc.out_rows,
-                          max_len=max(R) + steps)
-    ws = torch.empty(tb.tb_decode_workspace_size(ddesc), dtype=torch.uint8, device="cuda")
+    assert all(caps[b] >= R[b] + steps for b in range(B))
+    if check_at is None:
+        check_at = set(range(1, steps + 1)) if steps <= 16 else {1, 2, steps // 2, steps}
+
+    def ddesc(max_len):
+        return tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=DT[wl.dtype],
+                             cache_offset=desc.out_offset, cache_cap=caps, cache_rows=desc.out_rows,
+                             max_len=max_len)
+
+    last = ddesc(max(R) + steps)
+    ws_bytes = tb.tb_decode_workspace_size(last)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    tb.tb_decode_workspace_prepare(last, ws)
+    ws_ref = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
     Kc_t, Vc_t = res["Kc_t"], res["Vc_t"]
     out = torch.empty((B, wl.hq, wl.head_dim), dtype=torch.float32, device="cuda")
-    worst = 0.0
+    ref_out = torch.empty_like(out)
+    worst, layouts = 0.0, set()
     for s in range(1, steps + 1):
         st = inputs.make_decode_step(wl, layer, s, B)
         kn, vn = to_dev(st["k_new"], wl.dtype), to_dev(st["v_new"], wl.dtype)
@@ -94,10 +113,17 @@ def _decode_and_check(wl, lay, res, steps, heads_check=None, layer=0):
             Kc_t[:, row] = kn[:, b]
             Vc_t[:, row] = vn[:, b]
             lens.append(R[b] + s)
+        dd = ddesc(max(lens))
+        assert tb.tb_decode_workspace_size(dd) <= ws_bytes
+        layouts.add(tb.tb_decode_workspace_size(dd))
         lens_t = torch.tensor(lens, dtype=torch.int32, device="cuda")
         q_t = to_dev(st["q"], wl.dtype)
-        tb.tb_decode_attn(ddesc, q_t, Kc_t, Vc_t, lens_t, out, ws)
-        assert tb.tb_read_status(ws)[0] == tb.TB_OK
+        tb.tb_decode_attn_prepared(dd, q_t, Kc_t, Vc_t, lens_t, out, ws)
+        if s not in check_at:
+            continue
+        tb.tb_decode_attn(dd, q_t, Kc_t, Vc_t, lens_t, ref_out, ws_ref)
+        assert tb.tb_read_status(ws_ref)[0] == tb.TB_OK
+        assert torch.equal(out, ref_out), s
         got = out.cpu().numpy()
         Kc = _f32(wl, from_dev(Kc_t, wl.dtype))
         Vc = _f32(wl, from_dev(Vc_t, wl.dtype))
@@ -108,7 +134,8 @@ def _decode_and_check(wl, lay, res, steps, heads_check=None, layer=0):
             got, ref = got[:, hs], ref[:, hs]
         err = float(np.max(np.abs(got - ref)))
         worst = max(worst, err)
-        assert err <= TOL_OUT[wl.dtype], (s, err)
+        assert err <= TOL_OUT[wl.dtype], (s, lens, err)
+    assert tb.tb_read_status(ws) == (tb.TB_OK, 0)
     return worst
 
 
@@ -127,27 +154,34 @@ def test_tiny_config_evict_and_16_decode_steps():
     _decode_and_check(wl, lay, res, wl.decode_steps)
 
 
+@pytest.mark.parametrize("layer", [0, 27])
 @pytest.mark.parametrize("alpha", [0.0, 0.25, 0.5, 0.75])
-def test_7b_config(alpha):
+def test_7b_config(alpha, layer):
+    """First and last layer of the 28-layer stack at every alpha of the
+    workload, each followed by its 256-step decode loop."""
     wl = inputs.WORKLOADS["7b"]
-    lay = inputs.make_layer(wl, 3, alpha=alpha)
-    res = run_evict(wl, lay, extra_cap=4)
+    lay = inputs.make_layer(wl, layer, alpha=alpha)
+    res = run_evict(wl, lay, extra_cap=wl.decode_steps)
     ref = _oracle(wl, lay)
     _check_evict(wl, lay, res, ref)
-    _decode_and_check(wl, lay, res, 2, layer=3)
+    _decode_and_check(wl, lay, res, wl.decode_steps, layer=layer)
 
 
 def test_ragged_config():
+    """Every request of the 16-request batch, then the 256-step decode loop
+    over the ragged compacted caches."""
     wl = inputs.WORKLOADS["ragged"]
     lay = inputs.make_layer(wl, 5)
-    res = run_evict(wl, lay, extra_cap=2)
+    res = run_evict(wl, lay, extra_cap=wl.decode_steps)
     ref = _oracle(wl, lay)
     _check_evict(wl, lay, res, ref)
-    _decode_and_check(wl, lay, res, 2, layer=5)
+    _decode_and_check(wl, lay, res, wl.decode_steps, layer=5)
 
 
-def test_32k_config_alpha_sweep_sampled():
-    """Full-size 32K layer; the oracle scores once and selects per alpha."""
+def test_32k_config_alpha_sweep():
+    """Full-size 32K layer at all 20 alphas of the sweep (0.00 .. 0.95);
+    the oracle scores once and selects per alpha. Decode loops of the
+    workload's 512 steps follow the evictions at alpha 0, 0.5 and 0.95."""
     wl = inputs.WORKLOADS["32k"]
     lay = inputs.make_layer(wl, 0)
     dev = {k: to_dev(lay[k], wl.dtype) for k in ("q_win", "K", "V")}
@@ -156,26 +190,32 @@ def test_32k_config_alpha_sweep_sampled():
     S = orc.window_scores(q, K)
     pooled = orc.max_pool(S, wl.pool_k)
     n = int(lay["n"][0])
-    for alpha in (0.0, 0.05, 0.5, 0.9, 0.95):
+    assert len(wl.alpha_sweep) == 20
+    for alpha in wl.alpha_sweep:
         lay_a = dict(lay, alpha=np.array([alpha]))
-        res = run_evict(wl, lay_a, extra_cap=1, dev=dev)
+        res = run_evict(wl, lay_a, extra_cap=wl.decode_steps, dev=dev)
         k, R = orc.retained_count(n, wl.window, alpha)
         for g in range(wl.hkv):
             check_index_set(res["idx"][g, :R], pooled[g], k, n, wl.window)
             np.testing.assert_allclose(res["pooled"][g], pooled[g], rtol=TOL_SCORE_REL, atol=0)
-        if alpha == 0.5:
-            _decode_and_check(wl, lay_a, res, 1)
+            assert np.array_equal(from_dev(res["Kc_t"], wl.dtype)[g, :R], lay["K"][g, res["idx"][g, :R]])
+        if alpha in (0.0, 0.5, 0.95):
+            _decode_and_check(wl, lay_a, res, wl.decode_steps)
 
 
-def test_128k_config_sampled_heads():
-    """Full-size 128K layer in the launch configuration the benchmark times;
-    the oracle recomputes KV heads 0 and 7 only."""
+@pytest.mark.parametrize("layer", [0, 15, 31])
+def test_128k_config_sampled_heads(layer):
+    """Full-size 128K layers (first, middle, last of the 32) in the launch
+    configuration the benchmark times; the oracle recomputes KV heads 0 and
+    7. Layer 0 continues with the workload's 1024-step decode loop (lengths
+    13173 .. 14196), checked at steps 1, 2, 512 and 1024."""
     wl = inputs.WORKLOADS["128k"]
-    lay = inputs.make_layer(wl, 0)
-    res = run_evict(wl, lay, extra_cap=1)
+    lay = inputs.make_layer(wl, layer)
+    steps = wl.decode_steps if layer == 0 else 2
+    res = run_evict(wl, lay, extra_cap=steps)
     ref = _oracle(wl, lay, heads=[0, 7])
     _check_evict(wl, lay, res, ref, heads=[0, 7])
-    _decode_and_check(wl, lay, res, 1, heads_check=[0, 7])
+    _decode_and_check(wl, lay, res, steps, heads_check=[0, 7], layer=layer)
 
 
 # ---------------------------------------------------------------------------
@@ -365,21 +405,6 @@ def test_window_scores_stage():
     for b in range(2):
         s0, _, P, _ = request_slices(desc, b)
         np.testing.assert_allclose(got[:, s0:s0 + P], ref[b]["S"], rtol=TOL_SCORE_REL, atol=0)
-
-
-def test_fma_pipe_exp2_against_exact():
-    """The scoring epilogues' polynomial exponential: relative error below
-    2.2e-7 against exact 2^x (fp64) over [-125, 0.5], 2^-125 below that."""
-    x = np.concatenate([np.linspace(-125.0, 0.5, 2_000_001), np.linspace(-1.0, 0.0, 100_001),
-                        [0.0, -0.5, 0.5, -1.0, -124.99, -1000.0, -3e38]]).astype(np.float32)
-    xt = torch.from_numpy(x).cuda()
-    yt = torch.empty_like(xt)
-    tb.tb_diag_exp2(xt, yt)
-    y = yt.cpu().numpy().astype(np.float64)
-    xc = np.maximum(x.astype(np.float64), -125.0)
-    ref = np.exp2(xc)
-    rel = np.abs(y - ref) / ref
-    assert rel.max() < 2.2e-7, (rel.max(), x[np.argmax(rel)])
 
 
 @pytest.mark.parametrize("big", [False, True])
