@@ -429,3 +429,49 @@ def test_many_chunks_per_head_row_sums(big):
         s_max = float(np.max(inputs.as_f32(lay["q_win"], "bf16")[0, 0] @ inputs.as_f32(lay["K"], "bf16")[0, :64].T))
         assert s_max / np.sqrt(d) * np.log2(np.e) > 960
     _check_evict(wl, lay, res, ref)
+
+
+@pytest.mark.parametrize("d", [128, 64])
+@pytest.mark.parametrize("batch,hkv,G,lens", [
+    (1, 1, 8, [20000]),                       # one (request, KV head): several clusters, then a merge of their partials
+    (1, 8, 4, [13173]),                       # the 128K step's shape: one cluster per (request, KV head)
+    (20, 4, 7, [int(x) for x in np.random.default_rng(8).integers(0, 3000, 20)]),   # 80 units: the global merge
+])
+def test_decode_merge_forms(batch, hkv, G, lens, d):
+    """The decode's split merges on the layouts that select each of them on a
+    152-SM GB300 (clusters of 16 with several clusters per (request, KV
+    head); one cluster each; more (request, KV head) pairs than clusters fit,
+    so the splits merge through global memory), against the oracle, and
+    tb_decode_attn against tb_decode_attn_prepared bit for bit."""
+    rng = np.random.default_rng(batch * 31 + d)
+    hq = G * hkv
+    lens = list(lens)
+    lens[0] = max(lens[0], 1)
+    if batch > 2:
+        lens[1] = 0
+    caps = [x + 2 for x in lens]
+    offs = np.concatenate([[0], np.cumsum(caps)[:-1]]).astype(np.int64)
+    rows = int(np.sum(caps))
+    Kc = inputs.f32_to_bf16((rng.standard_normal((hkv, rows, d)) / np.sqrt(d)).astype(np.float32))
+    Vc = inputs.f32_to_bf16((rng.standard_normal((hkv, rows, d)) / np.sqrt(d)).astype(np.float32))
+    q = inputs.f32_to_bf16(rng.standard_normal((batch, hq, d)).astype(np.float32))
+    ddesc = tb.DecodeDesc(hq=hq, hkv=hkv, head_dim=d, dtype=tb.TB_BF16, cache_offset=offs, cache_cap=caps,
+                          cache_rows=rows, max_len=max(lens))
+    ws = torch.empty(tb.tb_decode_workspace_size(ddesc), dtype=torch.uint8, device="cuda")
+    wsp = torch.empty_like(ws)
+    tb.tb_decode_workspace_prepare(ddesc, wsp)
+    qd, Kd, Vd = to_dev(q, "bf16"), to_dev(Kc, "bf16"), to_dev(Vc, "bf16")
+    lens_t = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    out = torch.empty((batch, hq, d), dtype=torch.float32, device="cuda")
+    outp = torch.full_like(out, float("nan"))
+    tb.tb_decode_attn(ddesc, qd, Kd, Vd, lens_t, out, ws)
+    for _ in range(2):   # twice: the prepared workspace's counters are back at zero after a call
+        tb.tb_decode_attn_prepared(ddesc, qd, Kd, Vd, lens_t, outp, wsp)
+    assert tb.tb_read_status(ws) == (tb.TB_OK, 0) and tb.tb_read_status(wsp) == (tb.TB_OK, 0)
+    assert torch.equal(out, outp)
+    got = out.cpu().numpy()
+    ref = orc.decode_batch(inputs.as_f32(q, "bf16"), inputs.as_f32(Kc, "bf16"), inputs.as_f32(Vc, "bf16"),
+                           lens, offs)
+    assert np.max(np.abs(got - ref)) <= TOL_OUT["bf16"]
+    if batch > 2:
+        assert np.all(got[1] == 0)
