@@ -19,25 +19,13 @@
 //                  both multiplied by V (ldmatrix.trans) and accumulated in
 //                  fp32, so P enters with ~16 significant bits.
 // At the end the eight warps merge in shared memory into the split's partial
-// (max, sum, unnormalised output). The splits of a (request, KV head) then
-// merge in one of two ways:
-//  - cluster form: they run as thread-block clusters of C CTAs; every CTA
-//    keeps its partial in its own shared memory, and after a cluster barrier
-//    CTA r reads slice r of the outputs from all C partials through
-//    distributed shared memory (one round trip, no global memory). With more
-//    than one cluster per (request, KV head), each CTA writes its slice of
-//    the cluster's merged partial to the workspace and the last cluster to
-//    count in (a counter per slice) merges those;
-//  - global form (when clusters cannot be co-resident): every CTA writes its
-//    partial to the workspace and the CTA that finishes last among the
-//    (request, KV head)'s splits (a counter in the workspace: zero before the
-//    call, and set back to zero by that CTA) merges all splits.
+// (max, sum, unnormalised output); the CTA that finishes last among a
+// (request, KV head)'s splits (a counter in the workspace: zero before the
+// call, and set back to zero by that CTA) merges the splits and writes the
+// output.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
-
-#include <algorithm>
-#include <mutex>
 
 #include "tb_internal.cuh"
 #include "tc_ptx.cuh"
@@ -64,12 +52,6 @@ struct DGeo {
   static_assert(kMergeO + kWarps * 16 * 8 + 16 * kWarps * 4 <= kRing,
                 "merge area must fit in the ring");
   static constexpr int kMaxSplits = kRing / (16 * 4);  // weights table [G <= 16][splits]
-  // cluster form: the split's merged partial stays in shared memory for the
-  // cluster's other CTAs: O [16][D], (max, sum) [16], the CTA's ok flag
-  static constexpr int kCpoOff = (kMergeO + kWarps * 16 * 8 + 16 * kWarps * 4 + 15) / 16 * 16;
-  static constexpr int kCmlOff = kCpoOff + 16 * D * 4;
-  static constexpr int kCokOff = kCmlOff + 16 * 8;
-  static_assert(kCokOff + 16 <= kRing, "cluster partial must fit in the ring");
   static constexpr int kBarOff = kRing;
   static constexpr int kSmem = kBarOff + 64 + 1024;  // + alignment slack
 };
@@ -122,81 +104,7 @@ __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
   return (uint32_t)((chunk >> 3) * kBox + row * 128 + (((chunk & 7) ^ (row & 7)) << 4));
 }
 
-// Cluster form, after every CTA of the cluster wrote its split partial (O
-// unnormalised, (max, sum) per head, ok flag) into its own shared memory and
-// passed the first cluster barrier: CTA `rank` merges slice `rank` of the
-// G x D/4 float4 output groups over the cluster's C partials, reading them
-// through distributed shared memory. C lanes share a group (C divides 32),
-// one lane per split, and combine by shuffles. With one cluster per
-// (request, KV head) the result is the output; with more, the cluster's
-// merged partial for the slice goes to the workspace. Returns, through
-// *any_bad, whether some CTA of the cluster had aborted (then nothing is
-// written).
 template <int D, int G>
-__device__ __forceinline__ void cluster_merge(const DecodeParams& p, const float* cpo,
-                                              const float2* cml, const int* cok, uint32_t rank,
-                                              int unit, int cidx, int b, int g, void* out,
-                                              float* part_o, float2* part_ml) {
-  constexpr int D4 = D / 4;
-  constexpr int NG = G * D4;
-  const int C = p.cluster;
-  const int npg = (NG + C - 1) / C;
-  const int items = (npg * C + 31) & ~31;  // whole warps: every lane takes every shuffle
-  for (int it = threadIdx.x; it < items; it += kThreads) {
-    const int s = it % C, gl = it / C;
-    const int grp = (int)rank * npg + gl;
-    const bool valid = gl < npg && grp < NG;
-    const int h = valid ? grp / D4 : 0, d4 = valid ? grp % D4 : 0;
-    float2 ml = make_float2(-INFINITY, 0.f);
-    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-    int okv = 1;
-    if (valid) {
-      ml = tc::dsmem_ld_f2(tc::dsmem_addr(cml + h, (uint32_t)s));
-      o = tc::dsmem_ld_f4(tc::dsmem_addr(cpo + h * D + 4 * d4, (uint32_t)s));
-      okv = tc::dsmem_ld_s32(tc::dsmem_addr(cok, (uint32_t)s));
-    }
-    float M = ml.x;
-    for (int off = 1; off < C; off <<= 1) {
-      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-      okv &= __shfl_xor_sync(0xffffffffu, okv, off);
-    }
-    const float w = (ml.y > 0.f && M != -INFINITY) ? fast_exp2(ml.x - M) : 0.f;
-    float L = ml.y * w;
-    o.x *= w;
-    o.y *= w;
-    o.z *= w;
-    o.w *= w;
-    for (int off = 1; off < C; off <<= 1) {
-      L += __shfl_xor_sync(0xffffffffu, L, off);
-      o.x += __shfl_xor_sync(0xffffffffu, o.x, off);
-      o.y += __shfl_xor_sync(0xffffffffu, o.y, off);
-      o.z += __shfl_xor_sync(0xffffffffu, o.z, off);
-      o.w += __shfl_xor_sync(0xffffffffu, o.w, off);
-    }
-    if (s != 0 || !valid || !okv) continue;
-    if (p.clusters == 1) {
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-      const float4 r = make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv);
-      const size_t oi = ((size_t)b * p.hq + (size_t)g * G + h) * D + 4 * d4;
-      if (p.out_dtype == TB_F32) {
-        *reinterpret_cast<float4*>(static_cast<float*>(out) + oi) = r;
-      } else {
-        uint16_t* ob = static_cast<uint16_t*>(out) + oi;
-        ob[0] = float_to_bf16_rne(r.x);
-        ob[1] = float_to_bf16_rne(r.y);
-        ob[2] = float_to_bf16_rne(r.z);
-        ob[3] = float_to_bf16_rne(r.w);
-      }
-    } else {
-      // the cluster's partial of this group, relative to its max M
-      const size_t cb = (size_t)unit * p.clusters + cidx;
-      reinterpret_cast<float4*>(part_o)[cb * NG + grp] = o;
-      part_ml[cb * G + h] = make_float2(M, L);
-    }
-  }
-}
-
-template <int D, int G, bool kClu>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tma(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tk,
                const __grid_constant__ CUtensorMap tv, const uint16_t* __restrict__ q,
@@ -428,14 +336,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::mbar_wait(&full[s], (uint32_t)((last / kStages) & 1), &dummy, status);
       }
     }
-    // a cluster CTA still takes both cluster barriers (the others wait for
-    // it there), marked as aborted so that nothing is merged
-    if constexpr (!kClu) return;
+    return;
   }
-  float* cpo = reinterpret_cast<float*>(smem + Gm::kCpoOff);    // cluster form: [G][D]
-  float2* cml = reinterpret_cast<float2*>(smem + Gm::kCmlOff);  // [G]
-  int* cok = reinterpret_cast<int*>(smem + Gm::kCokOff);
-  if (ok) {
+
   // ---- merge the eight warps: O, m, l through shared memory (the ring is free)
 #pragma unroll
   for (int hr = 0; hr < 2; ++hr) {
@@ -481,10 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       wgt[h * kWarps + w] = wt;
       L = fmaf(mml[(w * 16 + h) * 2 + 1], wt, L);
     }
-    if constexpr (kClu)
-      cml[h] = make_float2(M, L);
-    else
-      part_ml[part_base + (size_t)h * p.splits] = make_float2(M, L);
+    part_ml[part_base + (size_t)h * p.splits] = make_float2(M, L);
   }
   __syncthreads();
   for (int e = tid; e < G * (D / 4); e += kThreads) {
@@ -499,74 +399,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       O.z = fmaf(ow.z, wt, O.z);
       O.w = fmaf(ow.w, wt, O.w);
     }
-    if constexpr (kClu)
-      *reinterpret_cast<float4*>(cpo + h * D + 4 * d4) = O;
-    else
-      *reinterpret_cast<float4*>(part_o + (part_base + (size_t)h * p.splits) * D + 4 * d4) = O;
-  }
-  }  // ok
-
-  if constexpr (kClu) {
-    // ---- cluster form: merge through distributed shared memory
-    if (tid == 0) *cok = ok ? 1 : 0;
-    const uint32_t rank = tc::cluster_ctarank();
-    const int unit = b * p.hkv + g, cidx = split / p.cluster;
-    tc::cluster_sync();  // every CTA's partial is in its shared memory
-    cluster_merge<D, G>(p, cpo, cml, cok, rank, unit, cidx, b, g, out, part_o, part_ml);
-    tc::cluster_sync();  // no CTA leaves while another still reads its partial
-    if (p.clusters == 1) return;
-    // ---- more than one cluster per (request, KV head): the last cluster to
-    // count in for this slice merges the clusters' partials of the slice. As
-    // in the global form, one thread counts the CTA in with an
-    // acquire-release atomic after a CTA barrier (which orders the slice's
-    // partial stores of every thread before it).
-    __syncthreads();
-    if (tid == 0) {
-      int* ctr = counters + (size_t)unit * kMaxDecodeCluster + rank;
-      int prev;
-      asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], 1;" : "=r"(prev) : "l"(ctr) : "memory");
-      *last_flag = prev == p.clusters - 1;
-      if (*last_flag) *ctr = 0;  // back to zero for the next call
-    }
-    __syncthreads();
-    if (!*last_flag) return;
-    constexpr int D4 = D / 4;
-    constexpr int NG = G * D4;
-    const int npg = (NG + p.cluster - 1) / p.cluster;
-    for (int gl = tid; gl < npg; gl += kThreads) {
-      const int grp = (int)rank * npg + gl;
-      if (grp >= NG) break;
-      const int h = grp / D4, d4 = grp % D4;
-      float M = -INFINITY;
-      for (int c = 0; c < p.clusters; ++c)
-        M = fmaxf(M, __ldcg(&part_ml[((size_t)unit * p.clusters + c) * G + h]).x);
-      float L = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int c = 0; c < p.clusters; ++c) {
-        const size_t cb = (size_t)unit * p.clusters + c;
-        const float2 ml = __ldcg(&part_ml[cb * G + h]);
-        const float w = (ml.y > 0.f && M != -INFINITY) ? fast_exp2(ml.x - M) : 0.f;
-        const float4 o = __ldcg(reinterpret_cast<const float4*>(part_o) + cb * NG + grp);
-        L = fmaf(ml.y, w, L);
-        acc.x = fmaf(o.x, w, acc.x);
-        acc.y = fmaf(o.y, w, acc.y);
-        acc.z = fmaf(o.z, w, acc.z);
-        acc.w = fmaf(o.w, w, acc.w);
-      }
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-      const size_t oi = ((size_t)b * p.hq + (size_t)g * G + h) * D + 4 * d4;
-      if (p.out_dtype == TB_F32) {
-        *reinterpret_cast<float4*>(static_cast<float*>(out) + oi) =
-            make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-      } else {
-        uint16_t* ob = static_cast<uint16_t*>(out) + oi;
-        ob[0] = float_to_bf16_rne(acc.x * inv);
-        ob[1] = float_to_bf16_rne(acc.y * inv);
-        ob[2] = float_to_bf16_rne(acc.z * inv);
-        ob[3] = float_to_bf16_rne(acc.w * inv);
-      }
-    }
-    return;
+    *reinterpret_cast<float4*>(part_o + (part_base + (size_t)h * p.splits) * D + 4 * d4) = O;
   }
 
   // ---- the last split CTA of this (request, KV head) merges every split.
@@ -579,13 +412,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     int prev;
     asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], 1;"
                  : "=r"(prev)
-                 : "l"(counters + (size_t)(b * p.hkv + g) * kMaxDecodeCluster)
+                 : "l"(counters + b * p.hkv + g)
                  : "memory");
     *last_flag = prev == p.splits - 1;
     // every split has counted in: the counter goes back to zero for the next
     // call (what a prepared workspace relies on; the clearing kernel of the
     // other entry points zeroes it anyway)
-    if (*last_flag) counters[(size_t)(b * p.hkv + g) * kMaxDecodeCluster] = 0;
+    if (*last_flag) counters[b * p.hkv + g] = 0;
   }
   __syncthreads();
   if (!*last_flag) return;
@@ -704,128 +537,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int D, int G, bool kClu>
+template <int D, int G>
 cudaError_t launch_g(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
                      const void* q, const int32_t* lens, float* part_o, float2* part_ml,
                      int32_t* counters, void* out, int32_t* status, cudaStream_t s) {
   using Gm = DGeo<D>;
-  auto kern = decode_tma<D, G, kClu>;
+  auto kern = decode_tma<D, G>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
-  if (kClu) {
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)p.splits, (unsigned)p.hkv, (unsigned)p.batch);
-  cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = Gm::kSmem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  int na = 0;
-  if (pdl_enabled()) {
-    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[na].val.programmaticStreamSerializationAllowed = 1;
-    ++na;
-  }
-  if (kClu) {
-    attr[na].id = cudaLaunchAttributeClusterDimension;
-    attr[na].val.clusterDim.x = (unsigned)p.cluster;
-    attr[na].val.clusterDim.y = 1;
-    attr[na].val.clusterDim.z = 1;
-    ++na;
-  }
-  cfg.attrs = attr;
-  cfg.numAttrs = na;
-  e = cudaLaunchKernelEx(&cfg, kern, p, tk, tv, static_cast<const uint16_t*>(q), lens, part_o, part_ml,
-                         counters, out, status);
+  e = launch_pdl(kern, dim3(p.splits, p.hkv, p.batch), dim3(kThreads), Gm::kSmem, s, p, tk, tv,
+                 static_cast<const uint16_t*>(q), lens, part_o, part_ml, counters, out, status);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
-}
-
-// Clusters of C CTAs of the cluster-form kernel that fit on the current
-// device at once (cudaOccupancyMaxActiveClusters; cached per device, 0 if
-// the query fails).
-template <int D, int G>
-int max_active_clusters(int C) {
-  constexpr int kMaxDev = 64;
-  static int cache[kMaxDev][5] = {};  // [device][log2 C], value + 1 once known
-  static std::mutex mu;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 0;
-  const int ci = C == 16 ? 4 : C == 8 ? 3 : C == 4 ? 2 : C == 2 ? 1 : 0;
-  if (ci == 0) return 0;
-  std::lock_guard<std::mutex> lock(mu);
-  if (cache[dev][ci] == 0) {
-    using Gm = DGeo<D>;
-    auto kern = decode_tma<D, G, true>;
-    int n = 0;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem) ==
-            cudaSuccess &&
-        cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
-            cudaSuccess) {
-      cudaLaunchConfig_t cfg = {};
-      cfg.gridDim = dim3((unsigned)C, 1, 1);
-      cfg.blockDim = dim3(kThreads, 1, 1);
-      cfg.dynamicSmemBytes = Gm::kSmem;
-      cudaLaunchAttribute attr;
-      attr.id = cudaLaunchAttributeClusterDimension;
-      attr.val.clusterDim.x = (unsigned)C;
-      attr.val.clusterDim.y = 1;
-      attr.val.clusterDim.z = 1;
-      cfg.attrs = &attr;
-      cfg.numAttrs = 1;
-      if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) n = 0;
-    }
-    (void)cudaGetLastError();  // a refused query leaves no sticky error
-    cache[dev][ci] = n + 1;
-  }
-  return cache[dev][ci] - 1;
-}
-
-// The cluster form's layout: the largest cluster size C (16, 8, 4, 2) of
-// which one cluster per (request, KV head) fits on the device at once, with
-// as many clusters M per (request, KV head) as fit (at least 64 keys per
-// split, at most the workspace's split count), taken as soon as the grid
-// covers 96 SMs or more, else the layout that covers the most. False when no
-// cluster size fits every (request, KV head) at once (the global form runs).
-template <int D, int G>
-bool plan_clusters(DecodeParams& p) {
-  const int64_t units = (int64_t)p.batch * p.hkv;
-  int bestC = 0, bestM = 0;
-  int64_t best_used = 0;
-  for (int C : {16, 8, 4, 2}) {
-    const int64_t q = max_active_clusters<D, G>(C);
-    if (q < units) continue;
-    int64_t M = std::min<int64_t>(q / units, std::max<int64_t>(1, p.max_len / (64 * C)));
-    M = std::max<int64_t>(1, std::min<int64_t>(M, p.splits));
-    const int64_t used = units * M * C;
-    if (used > best_used) {
-      bestC = C;
-      bestM = (int)M;
-      best_used = used;
-    }
-    if (used >= 96) break;
-  }
-  if (bestC == 0) return false;
-  p.cluster = bestC;
-  p.clusters = bestM;
-  p.splits = bestC * bestM;
-  int64_t split_len = (p.max_len + p.splits - 1) / p.splits;
-  p.split_len = (int32_t)((split_len + 15) / 16 * 16);
-  return true;
-}
-
-template <int D, int G>
-cudaError_t launch_gg(const DecodeParams& p0, const CUtensorMap& tk, const CUtensorMap& tv,
-                      const void* q, const int32_t* lens, float* part_o, float2* part_ml,
-                      int32_t* counters, void* out, int32_t* status, cudaStream_t s) {
-  DecodeParams p = p0;
-  if (plan_clusters<D, G>(p))
-    return launch_g<D, G, true>(p, tk, tv, q, lens, part_o, part_ml, counters, out, status, s);
-  p.cluster = 0;
-  p.clusters = 0;
-  return launch_g<D, G, false>(p, tk, tv, q, lens, part_o, part_ml, counters, out, status, s);
 }
 
 template <int D>
@@ -835,7 +558,7 @@ cudaError_t launch_d(const DecodeParams& p, const CUtensorMap& tk, const CUtenso
   switch (p.group) {
 #define TB_CASE(GG) \
   case GG:          \
-    return launch_gg<D, GG>(p, tk, tv, q, lens, part_o, part_ml, counters, out, status, s);
+    return launch_g<D, GG>(p, tk, tv, q, lens, part_o, part_ml, counters, out, status, s);
     TB_CASE(1) TB_CASE(2) TB_CASE(3) TB_CASE(4) TB_CASE(5) TB_CASE(6) TB_CASE(7) TB_CASE(8)
     TB_CASE(12) TB_CASE(16)
 #undef TB_CASE

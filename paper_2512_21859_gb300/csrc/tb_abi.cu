@@ -211,8 +211,8 @@ DecodeWorkspace carve_decode(const DecodeParams& p) {
   size_t off = 0;
   w.status = off;
   off += kStatusBytes;
-  w.counters = off;  // per (request, KV head): one per cluster rank
-  off = align_up(off + sizeof(int32_t) * (size_t)p.batch * p.hkv * kMaxDecodeCluster, 256);
+  w.counters = off;
+  off = align_up(off + sizeof(int32_t) * (size_t)p.batch * p.hkv, 256);
   w.part_o = off;
   off = align_up(off + sizeof(float) * (size_t)p.batch * p.hq * p.splits * p.d, 256);
   w.part_ml = off;

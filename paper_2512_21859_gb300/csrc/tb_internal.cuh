@@ -55,19 +55,9 @@ struct EvictParams {
   EvictReq req[TB_MAX_BATCH];
 };
 
-// Most CTAs of one thread-block cluster the decode uses (non-portable size),
-// and so the split counters each (request, KV head) keeps.
-constexpr int kMaxDecodeCluster = 16;
-
 struct DecodeParams {
   int32_t batch, hq, hkv, group, d, dtype, out_dtype, splits;
   int32_t split_len;  // keys per split
-  // thread-block clusters of the TMA decode: 0 = none (the last split CTA of
-  // a (request, KV head) merges all splits through global memory); C > 0 =
-  // the splits form clusters of C CTAs that merge through distributed shared
-  // memory, `clusters` of them per (request, KV head) (splits = C * clusters;
-  // with more than one cluster the last one merges the cluster partials)
-  int32_t cluster, clusters;
   // 1: the kernel just before the decode on the stream is the library's own
   // clearing kernel, so the first K/V tiles may be requested before the
   // dependency wait; 0 (prepared workspaces): anything may precede it

@@ -433,16 +433,15 @@ def test_many_chunks_per_head_row_sums(big):
 
 @pytest.mark.parametrize("d", [128, 64])
 @pytest.mark.parametrize("batch,hkv,G,lens", [
-    (1, 1, 8, [20000]),                       # one (request, KV head): several clusters, then a merge of their partials
-    (1, 8, 4, [13173]),                       # the 128K step's shape: one cluster per (request, KV head)
-    (20, 4, 7, [int(x) for x in np.random.default_rng(8).integers(0, 3000, 20)]),   # 80 units: the global merge
+    (1, 1, 8, [20000]),                       # one (request, KV head): 152 splits
+    (1, 8, 4, [13173]),                       # the 128K step's shape: 18 splits per (request, KV head)
+    (20, 4, 7, [int(x) for x in np.random.default_rng(8).integers(0, 3000, 20)]),   # 80 pairs, 2 splits each
 ])
-def test_decode_merge_forms(batch, hkv, G, lens, d):
-    """The decode's split merges on the layouts that select each of them on a
-    152-SM GB300 (clusters of 16 with several clusters per (request, KV
-    head); one cluster each; more (request, KV head) pairs than clusters fit,
-    so the splits merge through global memory), against the oracle, and
-    tb_decode_attn against tb_decode_attn_prepared bit for bit."""
+def test_decode_split_layouts(batch, hkv, G, lens, d):
+    """The decode's split merge on layouts from one (request, KV head) split
+    across the whole GPU to many pairs with two splits each (more CTAs than
+    fit at once), against the oracle, and tb_decode_attn against
+    tb_decode_attn_prepared bit for bit."""
     rng = np.random.default_rng(batch * 31 + d)
     hq = G * hkv
     lens = list(lens)
