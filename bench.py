@@ -303,9 +303,11 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
                         n=n, alpha=alpha_vec, kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)),
                         out_cap=lens_h)
     score_rows, idx_rows = tb.tb_evict_layout(desc)
+    # the step's own K/V row is in place before the decode, and the kernel
+    # before each decode writes no row of its cache: the early-read assertion holds
     ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
                           cache_offset=desc.out_offset, cache_cap=desc.out_cap,
-                          cache_rows=desc.out_rows, max_len=max(lens_h))
+                          cache_rows=desc.out_rows, max_len=max(lens_h), flags=tb.TB_DECODE_EARLY_CACHE_READ)
     ews = tb.tb_evict_workspace_size(desc)
     dws = tb.tb_decode_workspace_size(ddesc)
     step_in = inputs.make_decode_step(wl, rank, 1, B)
@@ -503,7 +505,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             "layers_rotated": L, "l2": "inputs larger than L2: %d rotating layer buffers of %.0f MB" % (
                 L, W["layer_bytes"] / 1e6),
             "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
-            "decode_call": "tb_decode_attn_prepared (workspace prepared once; no per-call clearing kernel)",
+            "decode_call": "tb_decode_attn_prepared with TB_DECODE_EARLY_CACHE_READ (workspace prepared once; "
+                           "no per-call clearing kernel; first tiles requested before the preceding kernel ends)",
             "launch": "each step is one CUDA-graph replay of the four C-ABI calls",
             "stage_timing": stage_timing,
             "parallelism": "replicas" if world > 1 else "single GPU"},

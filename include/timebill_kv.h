@@ -75,7 +75,7 @@ typedef enum { TB_F32 = 0, TB_BF16 = 1 } tb_dtype;
 /* Static description of a status code; never NULL. */
 const char *tb_status_string(int32_t status);
 
-/* Version of this ABI (major * 100 + minor). */
+/* Version of this ABI (major * 100 + minor): 101 (tb_decode_desc.flags). */
 int32_t tb_abi_version(void);
 
 /* Text of the last CUDA error this thread saw inside the library (the
@@ -209,6 +209,19 @@ tb_status tb_score_evict(const tb_evict_desc *desc, const void *q_win,
                          void *Kc, void *Vc, float *pooled, void *workspace,
                          size_t workspace_bytes, tb_stream_t stream);
 
+/* Bits of tb_decode_desc.flags. */
+/* The caller asserts that the work enqueued on the stream just before a
+ * tb_decode_attn_prepared call writes no row of Kc or Vc below lens[b] - 1
+ * (the row a decode loop appends last, lens[b] - 1, may be written by it;
+ * the rows before it were written earlier), and, if that work is a kernel
+ * using programmatic dependent launch, that it lets its successor start
+ * only after its own dependency wait. The decode kernel then requests its
+ * first K/V tiles before that work has completed (hiding their latency
+ * behind its tail) and reads row lens[b] - 1 again after it. No effect on
+ * tb_decode_attn and tb_decode_attn_noalloc, whose own clearing kernel
+ * already lets them do so. */
+#define TB_DECODE_EARLY_CACHE_READ 1
+
 /* Shape of one batched decode step. */
 typedef struct {
   int32_t batch;     /* 1 .. TB_MAX_BATCH */
@@ -221,6 +234,7 @@ typedef struct {
   const int64_t *cache_cap;    /* host [batch]: rows reserved for b */
   int64_t cache_rows;          /* rows per KV head of Kc and Vc */
   int64_t max_len;             /* upper bound of lens[b], >= 1 */
+  int32_t flags;               /* TB_DECODE_* bits; any other bit is an error */
 } tb_decode_desc;
 
 /* Bytes of device workspace tb_decode_attn needs for this descriptor. */

@@ -21,7 +21,7 @@ __all__ = [
     "TbError", "EvictDesc", "DecodeDesc", "library_path", "load",
     "tb_status_string", "tb_abi_version", "tb_last_error_detail", "tb_launch_counter",
     "tb_retained_count", "tb_retained_count_ex", "TB_EVICT_BUDGET_INCLUDES_WINDOW",
-    "TB_EVICT_AVG_POOL", "tb_evict_layout", "tb_evict_workspace_size",
+    "TB_EVICT_AVG_POOL", "TB_DECODE_EARLY_CACHE_READ", "tb_evict_layout", "tb_evict_workspace_size",
     "tb_window_scores", "tb_window_scores_lse", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
     "tb_decode_attn_noalloc", "tb_decode_noalloc_status", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_bounded_wait",
@@ -32,6 +32,7 @@ __all__ = [
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
 TB_F32, TB_BF16 = 0, 1
 TB_EVICT_BUDGET_INCLUDES_WINDOW, TB_EVICT_AVG_POOL = 1, 2
+TB_DECODE_EARLY_CACHE_READ = 1
 TB_MAX_BATCH = 64
 TB_NOALLOC_SCRATCH_BYTES = 4 << 20
 
@@ -54,7 +55,7 @@ class _DecodeDescC(ctypes.Structure):
         ("batch", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
         ("head_dim", ctypes.c_int32), ("dtype", ctypes.c_int32), ("out_dtype", ctypes.c_int32),
         ("cache_offset", _I64P), ("cache_cap", _I64P), ("cache_rows", ctypes.c_int64),
-        ("max_len", ctypes.c_int64),
+        ("max_len", ctypes.c_int64), ("flags", ctypes.c_int32),
     ]
 
 
@@ -217,13 +218,14 @@ class DecodeDesc:
     """tb_decode_desc plus its host arrays."""
 
     def __init__(self, *, hq: int, hkv: int, head_dim: int, dtype: int, cache_offset,
-                 cache_cap, cache_rows: int, max_len: int, out_dtype: int = TB_F32):
+                 cache_cap, cache_rows: int, max_len: int, out_dtype: int = TB_F32, flags: int = 0):
         self.cache_offset = np.ascontiguousarray(cache_offset, dtype=np.int64)
         self.cache_cap = np.ascontiguousarray(cache_cap, dtype=np.int64)
+        self.flags = int(flags)
         self.c = _DecodeDescC(
             int(self.cache_offset.shape[0]), hq, hkv, head_dim, dtype, out_dtype,
             self.cache_offset.ctypes.data_as(_I64P), self.cache_cap.ctypes.data_as(_I64P),
-            int(cache_rows), int(max_len))
+            int(cache_rows), int(max_len), self.flags)
         self.hq, self.hkv, self.head_dim, self.dtype, self.out_dtype = hq, hkv, head_dim, dtype, out_dtype
         self.cache_rows, self.max_len = int(cache_rows), int(max_len)
 

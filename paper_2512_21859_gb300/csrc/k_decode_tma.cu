@@ -107,7 +107,8 @@ __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
 template <int D, int G>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tma(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tk,
-               const __grid_constant__ CUtensorMap tv, const uint16_t* __restrict__ q,
+               const __grid_constant__ CUtensorMap tv, const uint16_t* __restrict__ kc,
+               const uint16_t* __restrict__ vc, const uint16_t* __restrict__ q,
                const int32_t* __restrict__ lens, float* __restrict__ part_o,
                float2* __restrict__ part_ml, int32_t* __restrict__ counters,
                void* __restrict__ out, int32_t* __restrict__ status) {
@@ -151,13 +152,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   };
   // With p.early_tma the first tiles are requested before the dependency
-  // wait: the kernel launched just before this one on the stream is then the
-  // library's own clearing kernel (it writes only the workspace's control
+  // wait. Mode 1: the kernel launched just before this one on the stream is
+  // the library's own clearing kernel (it writes only the workspace's control
   // words), which lets this one start only after its own wait has returned,
   // i.e. once every earlier kernel has completed and its writes are visible;
-  // the cache rows cannot be written by the clearing kernel. Without it (a
-  // prepared workspace, no clearing kernel) any kernel may precede this one,
-  // so the requests wait for it.
+  // the cache rows cannot be written by the clearing kernel. Mode 2: the
+  // caller asserts the same of the work before this kernel for every row
+  // below lens[b] - 1; that last row (appended by the decode loop, possibly
+  // by the preceding kernel) is read again after the wait, below. Without it
+  // (a prepared workspace, no assertion) any kernel may precede this one, so
+  // the requests wait for it.
   int issued = 0;
   if (tid == 0) {
     tc::tma_prefetch_desc(&tk);
@@ -178,6 +182,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int k1 = min(len, k0 + p.split_len);
   const int ntiles = k1 > k0 ? (k1 - k0 + kTile - 1) / kTile : 0;  // <= ntiles_c
   const size_t part_base = ((size_t)b * p.hq + (size_t)g * G) * p.splits + split;
+  // mode 2: the tile (one of those requested before the wait) holding the
+  // appended row len - 1, whose copy may predate the row; -1 if none
+  const int fresh_key = len - 1 - k0;
+  const int fresh_tile = (p.early_tma == 2 && fresh_key >= 0 && fresh_key < k1 - k0 &&
+                          fresh_key / kTile < kStages)
+                             ? fresh_key / kTile
+                             : -1;
 
   // Q fragments (rows >= G are zero queries)
   uint32_t aq[KS][4];
@@ -211,6 +222,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t kst = tc::smem_addr(smem + s * Gm::kStageBytes);
     const uint32_t vst = kst + (uint32_t)(Gm::KH * kBox);
     const int nvalid = min(kTile, k1 - (k0 + t * kTile));
+    if (t == fresh_tile) {
+      // the appended row, read again now that the kernel before this one has
+      // completed: the warp that owns it copies its K and V chunks over the
+      // tile's (swizzled) copy before reading them
+      const int row = fresh_key - t * kTile;
+      if ((row >> 4) == warp && lane < 2 * (D / 8)) {
+        const int half = lane / (D / 8), chunk = lane % (D / 8);
+        const size_t gi = ((size_t)g * p.cache_rows + p.cache_off[b] + (size_t)(k0 + fresh_key)) * D;
+        const uint4 v = __ldcg(reinterpret_cast<const uint4*>((half ? vc : kc) + gi) + chunk);
+        *reinterpret_cast<uint4*>(smem + s * Gm::kStageBytes + half * (Gm::KH * kBox) +
+                                  sw_off(row, chunk)) = v;
+      }
+      __syncwarp();
+    }
     if (kb < nvalid) {
       // rows past len may hold anything (even NaN): clear this warp's V rows there
       if (kb + 16 > nvalid) {
@@ -311,6 +336,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    // this stage's generic stores (the appended row, the cleared V rows)
+    // before the TMA refills it through the async proxy
+    if (t == fresh_tile || nvalid < kTile) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     __syncthreads();  // stage s is free again
     if (tid == 0 && issued < ntiles) {
       issue(issued);
@@ -539,13 +567,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int D, int G>
 cudaError_t launch_g(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
-                     const void* q, const int32_t* lens, float* part_o, float2* part_ml,
+                     const void* Kc, const void* Vc, const void* q, const int32_t* lens, float* part_o, float2* part_ml,
                      int32_t* counters, void* out, int32_t* status, cudaStream_t s) {
   using Gm = DGeo<D>;
   auto kern = decode_tma<D, G>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
   e = launch_pdl(kern, dim3(p.splits, p.hkv, p.batch), dim3(kThreads), Gm::kSmem, s, p, tk, tv,
+                 static_cast<const uint16_t*>(Kc), static_cast<const uint16_t*>(Vc),
                  static_cast<const uint16_t*>(q), lens, part_o, part_ml, counters, out, status);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
@@ -553,12 +582,12 @@ cudaError_t launch_g(const DecodeParams& p, const CUtensorMap& tk, const CUtenso
 
 template <int D>
 cudaError_t launch_d(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
-                     const void* q, const int32_t* lens, float* part_o, float2* part_ml,
+                     const void* Kc, const void* Vc, const void* q, const int32_t* lens, float* part_o, float2* part_ml,
                      int32_t* counters, void* out, int32_t* status, cudaStream_t s) {
   switch (p.group) {
 #define TB_CASE(GG) \
   case GG:          \
-    return launch_g<D, GG>(p, tk, tv, q, lens, part_o, part_ml, counters, out, status, s);
+    return launch_g<D, GG>(p, tk, tv, Kc, Vc, q, lens, part_o, part_ml, counters, out, status, s);
     TB_CASE(1) TB_CASE(2) TB_CASE(3) TB_CASE(4) TB_CASE(5) TB_CASE(6) TB_CASE(7) TB_CASE(8)
     TB_CASE(12) TB_CASE(16)
 #undef TB_CASE
@@ -586,8 +615,8 @@ cudaError_t launch_decode_tma(const DecodeParams& p, const void* q, const void* 
   if (!make_bf16_map(&tk, Kc, p.d, rows, kTile) || !make_bf16_map(&tv, Vc, p.d, rows, kTile))
     return cudaErrorInvalidValue;
   cudaError_t e =
-      p.d == 64 ? launch_d<64>(p, tk, tv, q, lens, part_o, part_ml, counters, out, status, s)
-                : launch_d<128>(p, tk, tv, q, lens, part_o, part_ml, counters, out, status, s);
+      p.d == 64 ? launch_d<64>(p, tk, tv, Kc, Vc, q, lens, part_o, part_ml, counters, out, status, s)
+                : launch_d<128>(p, tk, tv, Kc, Vc, q, lens, part_o, part_ml, counters, out, status, s);
   count_launches(1);
   return e;
 }

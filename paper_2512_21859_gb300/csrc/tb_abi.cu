@@ -161,6 +161,7 @@ tb_status check_ws(void* ws, size_t bytes, size_t need) {
 tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
   if (!d) return TB_ERR_INVALID_ARG;
   if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->max_len < 1) return TB_ERR_INVALID_ARG;
+  if ((d->flags & ~TB_DECODE_EARLY_CACHE_READ) != 0) return TB_ERR_INVALID_ARG;
   if (d->batch > TB_MAX_BATCH) return TB_ERR_UNSUPPORTED;
   if (d->hq % d->hkv != 0) return TB_ERR_INVALID_ARG;
   if (d->dtype != TB_F32 && d->dtype != TB_BF16) return TB_ERR_UNSUPPORTED;
@@ -319,7 +320,7 @@ const char* tb_status_string(int32_t status) {
   }
 }
 
-int32_t tb_abi_version(void) { return 100; }
+int32_t tb_abi_version(void) { return 101; }
 
 const char* tb_last_error_detail(void) { return g_last_error; }
 
@@ -617,8 +618,10 @@ tb_status tb_decode_attn_prepared(const tb_decode_desc* desc, const void* q, con
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   // no clearing kernel: the split counters are zero since the workspace was
   // prepared (each call's last split CTA zeroes its counter again), and the
-  // status word keeps what earlier calls raised
-  p.early_tma = 0;
+  // status word keeps what earlier calls raised. Any kernel may precede this
+  // one, so its first tiles wait for it, unless the caller asserts that the
+  // preceding work writes no cache row below the last appended one
+  p.early_tma = (desc->flags & TB_DECODE_EARLY_CACHE_READ) ? 2 : 0;
   return cuda_status(launch_decode(p, q, Kc, Vc, lens, out, at<float>(workspace, w.part_o),
                                    at<float2>(workspace, w.part_ml),
                                    at<int32_t>(workspace, w.counters),

@@ -60,7 +60,10 @@ struct DecodeParams {
   int32_t split_len;  // keys per split
   // 1: the kernel just before the decode on the stream is the library's own
   // clearing kernel, so the first K/V tiles may be requested before the
-  // dependency wait; 0 (prepared workspaces): anything may precede it
+  // dependency wait; 2: the same on the caller's word (prepared workspace
+  // with TB_DECODE_EARLY_CACHE_READ) that the work before it writes no cache
+  // row below lens[b] - 1, which is read again after the wait; 0 (prepared
+  // workspaces otherwise): anything may precede it
   int32_t early_tma;
   int64_t cache_rows;
   int64_t max_len;

@@ -43,7 +43,7 @@ def test_status_strings_and_version(tb):
     for s in range(6):
         assert tb.tb_status_string(s)
     assert tb.tb_status_string(99) == "unknown status"
-    assert tb.tb_abi_version() == 100
+    assert tb.tb_abi_version() == 101
     assert tb.tb_last_error_detail() == ""
 
 
@@ -161,6 +161,7 @@ def test_decode_workspace(tb):
     (dict(cache_rows=100), 1),
     (dict(cache_offset=[-4]), 1),
     (dict(hq=132, hkv=4), 2),                   # group of 33 heads at d=128
+    (dict(flags=2), 1),                         # an undefined flag bit
 ])
 def test_decode_desc_rejects(tb, kw, status):
     with pytest.raises(tb.TbError) as e:

@@ -98,3 +98,46 @@ def test_prepared_status_flag_is_sticky_until_prepared_again():
     assert np.max(np.abs(out.cpu().numpy() - want)) <= TOL_OUT["bf16"]
     tb.tb_decode_workspace_prepare(desc, ws)                 # prepared again: clear
     assert tb.tb_read_status(ws) == (tb.TB_OK, 0)
+
+
+@pytest.mark.parametrize("dtype,hq,hkv,d", [("bf16", 28, 4, 128), ("bf16", 32, 8, 128), ("bf16", 8, 1, 64)])
+def test_early_cache_read_in_a_decode_loop(dtype, hq, hkv, d):
+    """TB_DECODE_EARLY_CACHE_READ in the pattern it is for: every step first
+    appends its own K/V row at lens[b] - 1 (here with a copy kernel just
+    before the call), then runs tb_decode_attn_prepared with the flag, whose
+    kernel requests its first tiles before that copy has completed and reads
+    the appended row again after it. Bit-identical to tb_decode_attn on the
+    same cache at every step; the appended rows land in every position of a
+    tile (the lengths walk across tile and split boundaries)."""
+    caps = [700, 300, 2100]
+    offs, rows, q, Kc, Vc = _cache(hq * 3 + d, dtype, hq, hkv, d, caps)
+    rng = np.random.default_rng(d)
+    new_k = inputs.f32_to_bf16((rng.standard_normal((80, hkv, len(caps), d)) / np.sqrt(d)).astype(np.float32))
+    new_v = inputs.f32_to_bf16((rng.standard_normal((80, hkv, len(caps), d)) / np.sqrt(d)).astype(np.float32))
+    qd, Kd, Vd = to_dev(q, dtype), to_dev(Kc, dtype), to_dev(Vc, dtype)
+    nk, nv = to_dev(new_k, dtype), to_dev(new_v, dtype)
+    start = [600, 1, 1950]
+    base = dict(hq=hq, hkv=hkv, head_dim=d, dtype=DT[dtype], cache_offset=offs, cache_cap=caps, cache_rows=rows)
+    top = tb.DecodeDesc(max_len=max(caps), flags=tb.TB_DECODE_EARLY_CACHE_READ, **base)
+    ws = torch.empty(tb.tb_decode_workspace_size(top), dtype=torch.uint8, device="cuda")
+    tb.tb_decode_workspace_prepare(top, ws)
+    ws_ref = torch.empty_like(ws)
+    shape = (len(caps), hq, d)
+    out = torch.empty(shape, dtype=torch.float32, device="cuda")
+    ref = torch.empty(shape, dtype=torch.float32, device="cuda")
+    for step in range(80):
+        lens = [x + step for x in start]
+        for b in range(len(caps)):     # the step's own row, appended just before the call
+            Kd[:, offs[b] + lens[b] - 1] = nk[step, :, b]
+            Vd[:, offs[b] + lens[b] - 1] = nv[step, :, b]
+        lens_d = torch.tensor(lens, dtype=torch.int32, device="cuda")
+        flagged = tb.DecodeDesc(max_len=max(lens), flags=tb.TB_DECODE_EARLY_CACHE_READ, **base)
+        tb.tb_decode_attn_prepared(flagged, qd, Kd, Vd, lens_d, out, ws)
+        tb.tb_decode_attn(tb.DecodeDesc(max_len=max(lens), **base), qd, Kd, Vd, lens_d, ref, ws_ref)
+        assert torch.equal(out, ref), (step, lens)
+    assert tb.tb_read_status(ws) == (tb.TB_OK, 0)
+    got = out.cpu().numpy()
+    Kf = inputs.as_f32(Kd.view(torch.int16).cpu().numpy().view(np.uint16), dtype)
+    Vf = inputs.as_f32(Vd.view(torch.int16).cpu().numpy().view(np.uint16), dtype)
+    want = orc.decode_batch(inputs.as_f32(q, dtype), Kf, Vf, lens, offs)
+    assert np.max(np.abs(got - want)) <= TOL_OUT[dtype]

@@ -78,7 +78,8 @@ def _decode_and_check(wl, lay, res, steps, heads_check=None, layer=0, check_at=N
     (Eq. 8's N_kv^i grows by one row per step) and describes the step with
     max_len = the current longest length, so the split layout follows the
     lengths as they grow. The step runs through tb_decode_attn_prepared on
-    one workspace prepared before the loop (the call the benchmark times).
+    one workspace prepared before the loop, with the early cache read (the
+    call the benchmark times).
     At the steps in `check_at` (default: the first two, the middle and the
     last; every step for short loops) the output is compared with the
     oracle, and tb_decode_attn on the same inputs must give identical bits."""
@@ -91,9 +92,11 @@ def _decode_and_check(wl, lay, res, steps, heads_check=None, layer=0, check_at=N
         check_at = set(range(1, steps + 1)) if steps <= 16 else {1, 2, steps // 2, steps}
 
     def ddesc(max_len):
+        # the loop appends each step's row with its own copies just before the
+        # call and writes no other cache row: the early-read assertion holds
         return tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=DT[wl.dtype],
                              cache_offset=desc.out_offset, cache_cap=caps, cache_rows=desc.out_rows,
-                             max_len=max_len)
+                             max_len=max_len, flags=tb.TB_DECODE_EARLY_CACHE_READ)
 
     last = ddesc(max(R) + steps)
     ws_bytes = tb.tb_decode_workspace_size(last)
