@@ -299,6 +299,13 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
     for (int i = tid; i < cnt; i += kCsThreads) po[i] = __uint_as_float(keys[i]) * scale;
   }
 
+  // every prefix position kept (alpha = 0, or a budget above the prefix):
+  // the indices are the positions themselves, no selection or exchange
+  if (k >= P) {
+    for (int i = tid; i < cnt; i += kCsThreads) out[lo + i] = lo + i;
+    return;
+  }
+
   // ---- radix select of the k-th largest key (uniform across the cluster)
   unsigned tau = 0;
   int need = 0;
@@ -365,9 +372,6 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
       mask |= 255u << shift;
     }
     tau = prefix;
-  } else if (k >= P) {
-    tau = 0u;  // keep everything: every key is >= +0.0
-    need = P;
   }
 
   // ---- ordered compaction over warp-contiguous runs
