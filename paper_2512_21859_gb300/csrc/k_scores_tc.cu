@@ -15,7 +15,13 @@
 //  pass 2 (votes)       D[key][row] = K Q^T: each epilogue thread owns one key
 //                       (and a quarter of the rows) and sums 2^(t - c_row),
 //                       reading the key tiles in reverse order so that the
-//                       tail pass 1 loaded last is still in L2.
+//                       tail pass 1 loaded last is still in L2. The four
+//                       quarter sums of a key meet in global memory: the launch
+//                       that runs pass 1 clears the scores first, and each warp
+//                       adds its sum with a reduction (no hand-off between the
+//                       warps of a lane quadrant). The votes-only launch fed by
+//                       the prefill's log-sum-exp sums the quarters through
+//                       shared memory instead, in a fixed order.
 //
 // One kernel template runs pass 1, pass 2, or both. Both (the default) is a
 // cooperative launch of one CTA per SM: after pass 1 every CTA publishes its
@@ -65,7 +71,14 @@ constexpr int kSumMinChunks = 24;
 
 // kRowSums (with kPassBoth): the fp64 row sums replace the post-barrier
 // merge; a separate instantiation, so the kernel without it is unchanged
-enum : int { kPassStats = 1, kPassVotes = 2, kPassBoth = 3, kRowSums = 4 };
+// kRedVotes: the launch that runs pass 1 zeroes the scores as it starts, and
+// pass 2's warps add their quarter sums of the window rows into them with
+// global reductions (no hand-off between the four warps of a lane quadrant).
+// Measured on GB300 (128K, per call): 114.8 -> 108.7 us, with each warp's
+// reduction issued after its next TMEM load wait and relaxed hand-back
+// arrivals (issued before the wait, or behind a release arrival, the stores
+// stalled the warp: 134 us).
+enum : int { kPassStats = 1, kPassVotes = 2, kPassBoth = 3, kRowSums = 4, kRedVotes = 8 };
 
 template <int D>
 struct Geo {
@@ -248,6 +261,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const size_t segrow = ((size_t)info.b * p.hkv + info.g) * M;
   constexpr bool kFused = (MODE & kPassBoth) == kPassBoth;
   constexpr bool kSums = kFused && (MODE & kRowSums) != 0;
+  constexpr bool kRed = (MODE & kRedVotes) != 0;
+  float* const sc_out = scores + (size_t)info.g * p.score_rows + rq.score_off;
 
 
   // ---- set-up: barriers and the TMEM allocation
@@ -279,7 +294,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   // global memory from here on (the votes-only launch is a programmatic
   // dependent launch: its set-up above overlapped the previous kernel)
   pdl_wait();
-  if (MODE == kPassVotes) {
+  if (kRed && (MODE & kPassStats)) {
+    // the launch that runs pass 1 clears every score before any pass 2 tile
+    // adds into it (the grid barrier, or the launch boundary, orders the two);
+    // these stores go out while the first key tiles are on their way
+    const size_t total = (size_t)p.hkv * (size_t)p.score_rows;
+    const size_t per = (total + gridDim.x - 1) / gridDim.x;
+    const size_t z0 = per * blockIdx.x;
+    const int cnt = z0 < total ? (int)min(per, total - z0) : 0;
+    float* z = scores + z0;
+    for (int i = threadIdx.x; i < cnt; i += blockDim.x) z[i] = 0.f;
+  }
+  if ((MODE & kPassBoth) == kPassVotes) {
     for (int r = threadIdx.x; r < 256; r += blockDim.x)
       ncr[r] = r < M ? -(rowc[segrow + r] * p.rowc_scale) : -INFINITY;
     __syncthreads();
@@ -405,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // warp before computing, so the next-but-one tile's MMAs can start
           tc::tc_fence_before();
           __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
+          if (lane == 0) tc::mbar_arrive_rx(&bars->tempty[a]);
           released = true;
           if (!all_vis) {
 #pragma unroll
@@ -451,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!released) {
           tc::tc_fence_before();
           __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
+          if (lane == 0) tc::mbar_arrive_rx(&bars->tempty[a]);
         }
       }
       // the second column half hands its (max, sum) to the first
@@ -575,7 +601,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if ((MODE & kPassVotes) && ok) {
       // keys: TMEM lane quadrant quad; window rows (columns): quarter `sub`
       const int key = quad * 32 + lane;  // TMEM lane = key within the tile
-      float* out = scores + (size_t)info.g * p.score_rows + rq.score_off;
+      int pend_j = -1;  // a score store (or reduction) not yet issued
+      float pend_v = 0.f;
       for (int it2 = 0;; ++it2, ++it) {
         const int a = it & 1;
         if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) break;
@@ -594,9 +621,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::tmem_ld32(taddr + c0, *reinterpret_cast<float(*)[32]>(v));
           if (c0 + 32 < NP) tc::tmem_ld32(taddr + c0 + 32, *reinterpret_cast<float(*)[32]>(v + 32));
           tc::tmem_ld_wait();
+          // the previous tile's score store or reduction, issued after this
+          // wait (a TMEM load wait issued behind a global store waits for it)
+          if (pend_j >= 0) {
+            if (kRed) atomicAdd(sc_out + pend_j, pend_v);
+            else sc_out[pend_j] = pend_v;
+            pend_j = -1;
+          }
           tc::tc_fence_before();
           __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
+          if (lane == 0) tc::mbar_arrive_rx(&bars->tempty[a]);
           released = true;
           // 2^(v c - c_row) over the columns the MMA wrote: NP - c0 is a
           // multiple of 16, and columns past NP were never written
@@ -609,7 +643,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!released) {
           tc::tc_fence_before();
           __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->tempty[a]);
+          if (lane == 0) tc::mbar_arrive_rx(&bars->tempty[a]);
+        }
+        if (kRed) {
+          // this warp's quarter of the window rows, added into the key's score
+          const int j = t * kTileKeys + key;
+          if (sub * 64 < NP && j < rq.p) {
+            pend_j = j;
+            pend_v = acc;
+          }
+          continue;
         }
         // combine the four quarters of the window rows through a double-buffered
         // hand-off between the four warps of this lane quadrant (one SM
@@ -625,10 +668,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!tc::mbar_wait(&bars->xfull[x][quad], xph, abort, status)) break;
           const int j = t * kTileKeys + key;
           const float* xb = xbuf + x * 3 * 128;
-          if (j < rq.p) out[j] = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
+          if (j < rq.p) {
+            pend_j = j;
+            pend_v = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
+          }
           __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->xempty[x][quad]);
+          if (lane == 0) tc::mbar_arrive_rx(&bars->xempty[x][quad]);
         }
+      }
+      if (pend_j >= 0) {
+        if (kRed) atomicAdd(sc_out + pend_j, pend_v);
+        else sc_out[pend_j] = pend_v;
       }
     }
   }
@@ -698,7 +748,9 @@ cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const 
                             int32_t* tilectr, double* lsum, cudaStream_t s) {
   using Gm = Geo<D>;
   uint32_t* gsync = reinterpret_cast<uint32_t*>(status) + kGridSyncWord;
-  auto fused = window_scores_row_sums(pt) ? ws_tc<D, kPassBoth | kRowSums> : ws_tc<D, kPassBoth>;
+  constexpr int kRv = kRedVotes;
+  auto fused = window_scores_row_sums(pt) ? ws_tc<D, kPassBoth | kRowSums | kRv>
+                                          : ws_tc<D, kPassBoth | kRv>;
   cudaError_t e =
       cudaFuncSetAttribute(fused, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
@@ -720,8 +772,8 @@ cudaError_t launch_tc_typed(const EvictParams& pt, const CUtensorMap& tq, const 
     return cudaGetLastError();
   }
   // fallback: the passes as separate launches with the merge kernel between
-  auto stats = ws_tc<D, kPassStats>;
-  auto votes = ws_tc<D, kPassVotes>;
+  auto stats = ws_tc<D, kPassStats | kRv>;
+  auto votes = ws_tc<D, kPassVotes | kRv>;
   e = cudaFuncSetAttribute(stats, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(votes, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::kSmem);

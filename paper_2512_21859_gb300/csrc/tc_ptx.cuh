@@ -44,6 +44,15 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
+// An arrival that orders none of the thread's earlier memory accesses (a
+// release arrival waits until the thread's earlier global stores and
+// reductions are performed). For hand-backs whose data were already consumed:
+// an accumulator after tcgen05.wait::ld, a shared buffer whose values were used.
+__device__ __forceinline__ void mbar_arrive_rx(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar))
+               : "memory");
+}
+
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
                "r"(bytes)
