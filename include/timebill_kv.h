@@ -293,8 +293,17 @@ tb_status tb_decode_attn_prepared(const tb_decode_desc *desc, const void *q,
  * fired, e.g. a decode length above its cap). *raw (if not NULL) receives the
  * word itself. The word is cleared at the start of every call that can set
  * it: tb_window_scores, tb_score_evict and tb_decode_attn (tb_select_topk
- * and tb_gather_kv never set it and leave it as it was;
+ * never clears it and leaves it as it was; tb_gather_kv has no workspace;
  * tb_decode_attn_prepared keeps it until tb_decode_workspace_prepare).
+ *
+ * Debug build. libtimebill_kv_debug.so (the same entry points, built with
+ * TB_DEBUG=1) also checks, on the device, invariants the release kernels
+ * take for granted, and raises the same range bit (TB_ERR_INVALID_ARG here)
+ * when one fails instead of trapping: every window row's log-sum-exp is
+ * finite (non-finite inputs in q_win or K), tb_select_topk keeps exactly k
+ * positions, tb_score_evict's gather sees only indices in [0, N_b), and a
+ * decode head with keys has a positive finite softmax sum. The release
+ * library compiles these checks out.
  */
 tb_status tb_read_status(const void *workspace, size_t workspace_bytes,
                          tb_stream_t stream, int32_t *raw);

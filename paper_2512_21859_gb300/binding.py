@@ -72,7 +72,10 @@ class TbError(RuntimeError):
 
 
 def library_path() -> str:
-    return os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtimebill_kv.so")
+    """The release library, or with TB_LIBRARY=debug the TB_DEBUG build
+    (libtimebill_kv_debug.so, built by build.build(debug=True))."""
+    name = "libtimebill_kv_debug.so" if os.environ.get("TB_LIBRARY") == "debug" else "libtimebill_kv.so"
+    return os.path.join(os.path.dirname(os.path.abspath(__file__)), name)
 
 
 _LIB = None

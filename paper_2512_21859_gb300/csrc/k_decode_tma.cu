@@ -510,6 +510,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       L = fmaf(m2.y, wgt, L);
     }
     for (int off = 16; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
+    debug_flag(lane == 0 && len > 0 && !(L > 0.f && isfinite(L)), status);
     const float inv = L > 0.f ? 1.f / L : 0.f;
     __syncwarp();
     for (int sp = lane; sp < p.splits; sp += 32) wts[h * p.splits + sp] *= inv;

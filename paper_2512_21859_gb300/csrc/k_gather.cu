@@ -22,7 +22,7 @@ template <int VPR>
 __global__ void __launch_bounds__(kGatherThreads) gather_kernel(
     const __grid_constant__ EvictParams p, const int32_t* __restrict__ idx,
     const uint4* __restrict__ K, const uint4* __restrict__ V, uint4* __restrict__ Kc,
-    uint4* __restrict__ Vc) {
+    uint4* __restrict__ Vc, int32_t* __restrict__ status) {
   constexpr int kVecs = kRowsPerWarp * 2 * VPR;  // vectors a warp moves
   constexpr int kPerLane = kVecs / 32;
   static_assert(kPerLane <= kMaxVecPerLane, "too many vectors per lane");
@@ -47,6 +47,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(
     int j = -1;
     if (r < R) j = __ldg(ig + r);
     ok[i] = r < R && j >= 0 && j < rq.n;
+    debug_flag(r < R && !ok[i], status);  // an index outside the request's rows
     if (ok[i]) {
       const uint4* src = (w < VPR ? K : V) + src_base + (size_t)j * VPR + (w < VPR ? w : w - VPR);
       buf[i] = __ldg(src);
@@ -65,7 +66,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(
 }  // namespace
 
 cudaError_t launch_gather(const EvictParams& p, const int32_t* idx, const void* K,
-                          const void* V, void* Kc, void* Vc, cudaStream_t s) {
+                          const void* V, void* Kc, void* Vc, int32_t* status, cudaStream_t s) {
   const int elem = p.dtype == TB_F32 ? 4 : 2;
   const int vec_per_row = p.d * elem / 16;
   const int rows_per_block = (kGatherThreads / 32) * kRowsPerWarp;
@@ -78,9 +79,9 @@ cudaError_t launch_gather(const EvictParams& p, const int32_t* idx, const void* 
   uint4* vc4 = static_cast<uint4*>(Vc);
   cudaError_t e;
   switch (vec_per_row) {
-    case 8: e = launch_pdl(gather_kernel<8>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4); break;
-    case 16: e = launch_pdl(gather_kernel<16>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4); break;
-    case 32: e = launch_pdl(gather_kernel<32>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4); break;
+    case 8: e = launch_pdl(gather_kernel<8>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4, status); break;
+    case 16: e = launch_pdl(gather_kernel<16>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4, status); break;
+    case 32: e = launch_pdl(gather_kernel<32>, grid, dim3(kGatherThreads), 0, s, p, idx, k4, v4, kc4, vc4, status); break;
     default: return cudaErrorInvalidValue;
   }
   count_launches(1);

@@ -308,6 +308,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if ((MODE & kPassBoth) == kPassVotes) {
     for (int r = threadIdx.x; r < 256; r += blockDim.x)
       ncr[r] = r < M ? -(rowc[segrow + r] * p.rowc_scale) : -INFINITY;
+    debug_flag(threadIdx.x < M && !isfinite(ncr[threadIdx.x]), status);
     __syncthreads();
   }
   // (no early pdl_trigger here: the select's CTAs launched during the scoring
@@ -554,6 +555,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                            0x3ff0000000000000LL);
             v = -((float)e + log2f(mant));
           }
+          debug_flag(r < M && !isfinite(v), status);  // a row normaliser out of range
           ncr[r] = v;
         }
       } else if (ok) {
@@ -590,6 +592,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float ll = (l > 0.f ? l * exp2f(m - mm) : 0.f) + (lo > 0.f ? lo * exp2f(mo - mm) : 0.f);
             v = -(mm + log2f(ll));
           }
+          debug_flag(r < M && !isfinite(v), status);  // a row normaliser out of range
           ncr[r] = v;
         }
       }

@@ -68,7 +68,8 @@ __device__ __forceinline__ int block_scan_flag(bool flag, int* warp_tot, int* to
 
 __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ EvictParams p,
                                                              const float* __restrict__ pooled,
-                                                             int32_t* __restrict__ idx) {
+                                                             int32_t* __restrict__ idx,
+                                                             int32_t* __restrict__ status) {
   __shared__ unsigned hist[256];
   __shared__ int warp_tot[33];
   __shared__ unsigned sh_prefix;
@@ -150,9 +151,11 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     int tot_sel;
     const int pos = base_sel + block_scan_flag(sel, warp_tot, &tot_sel);
     if (sel && pos < k) out[pos] = j;
+    debug_flag(sel && pos >= k, status);
     base_sel += tot_sel;
     base_tie += tot_eq;
   }
+  debug_flag(tid == 0 && base_sel != k, status);  // exactly k positions kept
 }
 
 
@@ -181,7 +184,8 @@ struct ClusterSelectShared {
 
 __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
     const __grid_constant__ EvictParams p, const float* __restrict__ scores,
-    float* __restrict__ pooled_out, int32_t* __restrict__ idx, int slice) {
+    float* __restrict__ pooled_out, int32_t* __restrict__ idx, int32_t* __restrict__ status,
+    int slice) {
   namespace cg = cooperative_groups;
   cg::cluster_group cluster = cg::this_cluster();
   __shared__ ClusterSelectShared sh;
@@ -450,11 +454,15 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
         const unsigned sm = __ballot_sync(0xffffffffu, sel);
         const int pos = selbase + __popc(sm & lt);
         if (sel && pos < k) out[pos] = lo + i;
+        debug_flag(sel && pos >= k, status);
         selbase += __popc(sm);
         eqbase += __popc(em);
       }
     }
   }
+  // the cluster's last warp ends on the total: exactly k positions kept
+  debug_flag(k > 0 && rank == cs - 1 && warp == kCsWarps - 1 && lane == 0 && selbase != k,
+             status);
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
@@ -470,8 +478,8 @@ cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled
 }
 
 cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* idx,
-                          cudaStream_t s) {
-  select_kernel<<<p.batch * p.hkv, kSelThreads, 0, s>>>(p, pooled, idx);
+                          int32_t* status, cudaStream_t s) {
+  select_kernel<<<p.batch * p.hkv, kSelThreads, 0, s>>>(p, pooled, idx, status);
   count_launches(1);
   return cudaGetLastError();
 }
@@ -491,7 +499,7 @@ int select_cluster_size(const EvictParams& p) {
 }
 
 cudaError_t launch_select_cluster(const EvictParams& p, const float* scores, float* pooled_out,
-                                  int32_t* idx, cudaStream_t s) {
+                                  int32_t* idx, int32_t* status, cudaStream_t s) {
   const int cs = select_cluster_size(p);
   const int slice = (p.max_p + cs - 1) / cs;
   // slice + halo, plus slack for the grouped max-pool's last 16-byte loads
@@ -513,7 +521,7 @@ cudaError_t launch_select_cluster(const EvictParams& p, const float* scores, flo
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl_enabled() ? 2 : 1;
-  e = cudaLaunchKernelEx(&cfg, select_cluster_kernel, p, scores, pooled_out, idx, slice);
+  e = cudaLaunchKernelEx(&cfg, select_cluster_kernel, p, scores, pooled_out, idx, status, slice);
   count_launches(1);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

@@ -13,9 +13,18 @@
 #include <vector>
 #include <atomic>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "tb_internal.cuh"
 
 namespace tb {
+
+// A named NVTX range around a compute entry point (its host-side launch
+// sequence), for timeline tools: ncu --nvtx, Nsight Systems. Without a tool
+// attached a range costs a function-pointer check.
+NvtxRange::NvtxRange(const char* name) { nvtxRangePushA(name); }
+NvtxRange::~NvtxRange() { nvtxRangePop(); }
+
 namespace {
 
 thread_local char g_last_error[256] = "";
@@ -244,10 +253,12 @@ tb_status run_window_scores(const EvictParams& p, const EvictWorkspace& w, const
 
 tb_status run_select(const EvictParams& p, const EvictWorkspace& w, const float* scores,
                      int32_t* idx, float* pooled, void* ws, cudaStream_t s) {
-  if (select_cluster_supported(p)) return cuda_status(launch_select_cluster(p, scores, pooled, idx, s));
+  int32_t* status = at<int32_t>(ws, w.status);
+  if (select_cluster_supported(p))
+    return cuda_status(launch_select_cluster(p, scores, pooled, idx, status, s));
   float* pl = pooled ? pooled : at<float>(ws, w.pooled);
   cudaError_t e = launch_pool(p, scores, pl, s);
-  if (e == cudaSuccess) e = launch_select(p, pl, idx, s);
+  if (e == cudaSuccess) e = launch_select(p, pl, idx, status, s);
   return cuda_status(e);
 }
 
@@ -488,6 +499,7 @@ tb_status tb_evict_workspace_size(const tb_evict_desc* desc, size_t* bytes) {
 tb_status tb_window_scores(const tb_evict_desc* desc, const void* q_win, const void* K,
                            float* scores, void* workspace, size_t workspace_bytes,
                            tb_stream_t stream) {
+  const NvtxRange range("tb_window_scores");
   EvictParams p;
   tb_status st = build_evict(desc, &p);
   if (st != TB_OK) return st;
@@ -503,6 +515,7 @@ tb_status tb_window_scores(const tb_evict_desc* desc, const void* q_win, const v
 tb_status tb_window_scores_lse(const tb_evict_desc* desc, const void* q_win, const void* K,
                                const float* lse, float* scores, void* workspace,
                                size_t workspace_bytes, tb_stream_t stream) {
+  const NvtxRange range("tb_window_scores_lse");
   EvictParams p;
   tb_status st = build_evict(desc, &p);
   if (st != TB_OK) return st;
@@ -521,6 +534,7 @@ tb_status tb_window_scores_lse(const tb_evict_desc* desc, const void* q_win, con
 tb_status tb_select_topk(const tb_evict_desc* desc, const float* scores, int32_t* idx,
                          float* pooled, void* workspace, size_t workspace_bytes,
                          tb_stream_t stream) {
+  const NvtxRange range("tb_select_topk");
   EvictParams p;
   tb_status st = build_evict(desc, &p);
   if (st != TB_OK) return st;
@@ -536,6 +550,7 @@ tb_status tb_select_topk(const tb_evict_desc* desc, const float* scores, int32_t
 
 tb_status tb_gather_kv(const tb_evict_desc* desc, const int32_t* idx, const void* K,
                        const void* V, void* Kc, void* Vc, tb_stream_t stream) {
+  const NvtxRange range("tb_gather_kv");
   EvictParams p;
   const tb_status st = build_evict(desc, &p);
   if (st != TB_OK) return st;
@@ -543,12 +558,13 @@ tb_status tb_gather_kv(const tb_evict_desc* desc, const int32_t* idx, const void
   if (!aligned16(idx) || !aligned16(K) || !aligned16(V) || !aligned16(Kc) || !aligned16(Vc))
     return TB_ERR_INVALID_ARG;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  return cuda_status(launch_gather(p, idx, K, V, Kc, Vc, s));
+  return cuda_status(launch_gather(p, idx, K, V, Kc, Vc, nullptr, s));
 }
 
 tb_status tb_score_evict(const tb_evict_desc* desc, const void* q_win, const void* K,
                          const void* V, int32_t* idx, void* Kc, void* Vc, float* pooled,
                          void* workspace, size_t workspace_bytes, tb_stream_t stream) {
+  const NvtxRange range("tb_score_evict");
   EvictParams p;
   tb_status st = build_evict(desc, &p);
   if (st != TB_OK) return st;
@@ -563,7 +579,7 @@ tb_status tb_score_evict(const tb_evict_desc* desc, const void* q_win, const voi
   float* scores = at<float>(workspace, w.scores);
   if ((st = run_window_scores(p, w, q_win, K, scores, workspace, s)) != TB_OK) return st;
   if ((st = run_select(p, w, scores, idx, pooled, workspace, s)) != TB_OK) return st;
-  return cuda_status(launch_gather(p, idx, K, V, Kc, Vc, s));
+  return cuda_status(launch_gather(p, idx, K, V, Kc, Vc, at<int32_t>(workspace, w.status), s));
 }
 
 tb_status tb_decode_workspace_size(const tb_decode_desc* desc, size_t* bytes) {
@@ -578,6 +594,7 @@ tb_status tb_decode_workspace_size(const tb_decode_desc* desc, size_t* bytes) {
 tb_status tb_decode_attn(const tb_decode_desc* desc, const void* q, const void* Kc,
                          const void* Vc, const int32_t* lens, void* out, void* workspace,
                          size_t workspace_bytes, tb_stream_t stream) {
+  const NvtxRange range("tb_decode_attn");
   DecodeParams p;
   tb_status st = build_decode(desc, &p);
   if (st != TB_OK) return st;
@@ -596,6 +613,7 @@ tb_status tb_decode_attn(const tb_decode_desc* desc, const void* q, const void* 
 
 tb_status tb_decode_workspace_prepare(const tb_decode_desc* desc, void* workspace,
                                       size_t workspace_bytes, tb_stream_t stream) {
+  const NvtxRange range("tb_decode_workspace_prepare");
   DecodeParams p;
   tb_status st = build_decode(desc, &p);
   if (st != TB_OK) return st;
@@ -608,6 +626,7 @@ tb_status tb_decode_workspace_prepare(const tb_decode_desc* desc, void* workspac
 tb_status tb_decode_attn_prepared(const tb_decode_desc* desc, const void* q, const void* Kc,
                                   const void* Vc, const int32_t* lens, void* out, void* workspace,
                                   size_t workspace_bytes, tb_stream_t stream) {
+  const NvtxRange range("tb_decode_attn_prepared");
   DecodeParams p;
   tb_status st = build_decode(desc, &p);
   if (st != TB_OK) return st;

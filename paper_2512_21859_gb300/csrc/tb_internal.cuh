@@ -100,6 +100,13 @@ bool make_bf16_map(CUtensorMap* map, const void* base, int d, uint64_t rows, int
 // Adds n to the process-wide launch counter (tb_launch_counter).
 void count_launches(int n);
 
+struct NvtxRange {
+  explicit NvtxRange(const char* name);
+  ~NvtxRange();
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 // Programmatic dependent launch. A kernel launched by launch_pdl may begin
 // (its CTAs made resident, their set-up run) while the previous kernel of the
 // stream is still finishing: it calls pdl_wait() before its first access to
@@ -167,15 +174,16 @@ cudaError_t launch_window_scores_tc(const EvictParams& p, const void* q_win, con
 cudaError_t launch_pool(const EvictParams& p, const float* scores, float* pooled,
                         cudaStream_t s);
 cudaError_t launch_select(const EvictParams& p, const float* pooled, int32_t* idx,
-                          cudaStream_t s);
+                          int32_t* status, cudaStream_t s);
 // Cluster select with the max-pool fused in (pooled_out may be null).
 constexpr int kClusterSliceMax = 16 * 1024;  // keys per CTA: 16 per thread of 1024
 int select_cluster_size(const EvictParams& p);
 bool select_cluster_supported(const EvictParams& p);
 cudaError_t launch_select_cluster(const EvictParams& p, const float* scores, float* pooled_out,
-                                  int32_t* idx, cudaStream_t s);
+                                  int32_t* idx, int32_t* status, cudaStream_t s);
+// status may be null (tb_gather_kv has no workspace)
 cudaError_t launch_gather(const EvictParams& p, const int32_t* idx, const void* K,
-                          const void* V, void* Kc, void* Vc, cudaStream_t s);
+                          const void* V, void* Kc, void* Vc, int32_t* status, cudaStream_t s);
 // TMA-staged bf16 decode (split partials only; the caller launches the combine).
 bool decode_tma_supported(const DecodeParams& p);
 cudaError_t launch_decode_tma(const DecodeParams& p, const void* q, const void* Kc,
@@ -189,6 +197,21 @@ cudaError_t launch_decode(const DecodeParams& p, const void* q, const void* Kc,
 // ---------------------------------------------------------------------------
 // device helpers
 // ---------------------------------------------------------------------------
+// Debug builds (TB_DEBUG=1, libtimebill_kv_debug.so) check invariants the
+// release kernels take for granted (index ranges, finite normalisers, the
+// selected count) and raise kStatusRange in the status word when one fails,
+// instead of trapping; release builds compile the checks out.
+#ifndef TB_DEBUG
+#define TB_DEBUG 0
+#endif
+__device__ __forceinline__ void debug_flag(bool bad, int32_t* status) {
+#if TB_DEBUG
+  if (bad && status) atomicOr(status, kStatusRange);
+#else
+  (void)bad;
+  (void)status;
+#endif
+}
 __device__ __forceinline__ float bf16_bits_to_float(uint16_t v) {
   return __uint_as_float(static_cast<uint32_t>(v) << 16);
 }
