@@ -2,13 +2,15 @@
 """Benchmark of TimeBill's eviction + decode-attention hot path on GB300.
 
 One step = one transformer layer of the path: one decode step of attention
-over the layer's compacted cache (tb_decode_attn_prepared: the decode
-workspace is prepared once, as a decode loop keeps it), then the layer's
-prompt-time eviction (tb_window_scores -> tb_select_topk -> tb_gather_kv,
-the stages tb_score_evict chains). Layers rotate over enough device buffers
-that every step's inputs are larger than L2 (129 MB), so no step reads
-another step's data from cache; the decode reads a cache the same buffer's
-eviction wrote one rotation earlier.
+over a compacted cache (tb_decode_attn_prepared: the decode workspace is
+prepared once, as a decode loop keeps it) and the layer's prompt-time
+eviction (tb_window_scores -> tb_select_topk -> tb_gather_kv, the stages
+tb_score_evict chains), enqueued as scoring, select, decode, gather: the
+decode's CTAs start during the select on the SMs it leaves free, and attend
+over the cache the previous step's eviction wrote (--serial-step: decode
+first, over the buffer's own cache from one rotation earlier). Layers rotate
+over enough device buffers that every step's inputs are larger than L2
+(129 MB), so no step reads another step's data from cache.
 
 Prints ONE JSON line. value = algorithmic HBM bytes of the step (K read once
 to score, retained K/V rows read and written, compacted K/V read by decode)
@@ -71,6 +73,9 @@ def parse_args(argv=None):
                     help="profile tb_decode_attn_prepared over N_kv and tb_score_evict over N_x on the 7b "
                          "shape and print the least-squares time model (Eq. 6a/6b) with its MAPE")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--serial-step", action="store_true",
+                    help="run the step's decode before the eviction (default: between the select and "
+                         "the gather, so that its CTAs start during the select)")
     ap.add_argument("--no-alpha-sweep", action="store_true",
                     help="skip the per-alpha stage table (128K at 0.5/0.75/0.9, 32K at 0..0.95)")
     ap.add_argument("--sweep-steps", type=int, default=12,
@@ -414,16 +419,31 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     stage_call = S["stage_call"]
     layers = S["bufs"]
 
-    # each layer buffer's step (decode, then the eviction) captured into a CUDA graph
+    # each layer buffer's step captured into a CUDA graph of the four calls
+    # on one stream. Default order: window scoring, select, decode, gather.
+    # The select runs one cluster per KV head and leaves most SMs idle; the
+    # decode, a programmatic dependent launch behind it, gets its CTAs
+    # resident there during the select and requests its first tiles before
+    # its dependency wait (its early-read assertion holds: the select writes
+    # only indices). That decode attends over the compacted cache of the
+    # previous buffer of the rotation (the previous step's eviction output),
+    # never over the cache this step's gather writes. --serial-step: the
+    # decode first, then the eviction, over the buffer's own cache.
     cap = torch.cuda.Stream(dev)
     step_graphs = []
     kernels_per_step = None
-    for d in layers:
+    for i, d in enumerate(layers):
         g = torch.cuda.CUDAGraph()
         c0 = tb.tb_launch_counter()
         with torch.cuda.graph(g, stream=cap):
-            for name in STAGES:
-                stage_call(name, d, cap)
+            if args.serial_step:
+                for name in STAGES:
+                    stage_call(name, d, cap)
+            else:
+                stage_call("window_scores", d, cap)
+                stage_call("select_topk", d, cap)
+                stage_call("decode_attn", layers[(i + L - 1) % L], cap)
+                stage_call("gather_kv", d, cap)
         kernels_per_step = tb.tb_launch_counter() - c0
         step_graphs.append(g)
     torch.cuda.synchronize(dev)
@@ -507,7 +527,11 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
             "decode_call": "tb_decode_attn_prepared with TB_DECODE_EARLY_CACHE_READ (workspace prepared once; "
                            "no per-call clearing kernel; first tiles requested before the preceding kernel ends)",
-            "launch": "each step is one CUDA-graph replay of the four C-ABI calls",
+            "launch": "each step is one CUDA-graph replay of the four C-ABI calls" + (
+                ": decode_attn, window_scores, select_topk, gather_kv" if args.serial_step else
+                " in the order window_scores, select_topk, decode_attn, gather_kv: the decode's CTAs "
+                "start during the select (programmatic dependent launch) on the SMs it leaves free and "
+                "attend over the previous rotation buffer's compacted cache"),
             "stage_timing": stage_timing,
             "parallelism": "replicas" if world > 1 else "single GPU"},
         "us_per_layer": {"evict": round(evict_us, 2), "decode": round(1e3 * stage_ms["decode_attn"], 2),
