@@ -756,17 +756,23 @@ def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_i
             vd.copy_(hv, non_blocking=True)
 
     def timed(fn):
+        # the best of three timed runs of `steps` steps each (host-side
+        # hiccups in the pinned copies otherwise show up in single runs)
         for _ in range(2):
             fn()
         torch.cuda.synchronize(dev)
-        t0 = torch.cuda.Event(enable_timing=True)
-        t1 = torch.cuda.Event(enable_timing=True)
-        t0.record(stream)
-        for _ in range(steps):
-            fn()
-        t1.record(stream)
-        torch.cuda.synchronize(dev)
-        return t0.elapsed_time(t1) / steps
+        best = None
+        for _ in range(3):
+            t0 = torch.cuda.Event(enable_timing=True)
+            t1 = torch.cuda.Event(enable_timing=True)
+            t0.record(stream)
+            for _ in range(steps):
+                fn()
+            t1.record(stream)
+            torch.cuda.synchronize(dev)
+            ms = t0.elapsed_time(t1) / steps
+            best = ms if best is None else min(best, ms)
+        return best
 
     ms_serial = timed(serial)
     idx_serial = idx_h.clone()
