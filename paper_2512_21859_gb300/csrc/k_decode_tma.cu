@@ -38,6 +38,10 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kTile = kWarps * 16;  // keys per tile: 16 per warp
 constexpr int kStages = 3;          // one CTA per SM, 3 x 64 KB in flight
 constexpr int kBox = kTile * 128;   // one TMA box: kTile rows x 128 B
+#ifndef TB_MERGE_PARTS
+#define TB_MERGE_PARTS 4
+#endif
+constexpr int kMergeParts = TB_MERGE_PARTS;  // CTAs of the merge kernel per (KV head, request)
 
 template <int D>
 struct DGeo {
@@ -102,6 +106,133 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 // inside a stage half (K or V) laid out as KH boxes of 64 rows x 128 B, 128B-swizzled
 __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
   return (uint32_t)((chunk >> 3) * kBox + row * 128 + (((chunk & 7) ^ (row & 7)) << 4));
+}
+
+// Merges the key splits of (request b, KV head g) into the output: per head
+// the weight 2^(m_s - M) / L of every split s, then each output element as
+// one pass over the splits' unnormalised partial outputs: the dims of part
+// `dpart` of DS equal parts. wts: shared memory for [G][splits] floats.
+template <int D, int G, int DS>
+__device__ __forceinline__ void merge_splits(const DecodeParams& p, int b, int g, int dpart,
+                                             const float* __restrict__ part_o,
+                                             const float2* __restrict__ part_ml,
+                                             void* __restrict__ out, int32_t* __restrict__ status,
+                                             float* wts, int len) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const size_t head0 = ((size_t)b * p.hq + (size_t)g * G) * p.splits;
+  // outputs in float4 groups of dims; the splits are divided among the
+  // threads that share an output (NS of them), their sums combined by shuffles
+  constexpr int D4 = D / 4 / DS;  // float4 groups of this part
+  const int d4_0 = dpart * D4;
+  // (G * D4 * NS is a multiple of 32 for every supported G and D, so each
+  // warp's lanes run the same iterations and the shuffles see full warps)
+  constexpr int kPer = kThreads / (G * D4);
+  constexpr int NS = kPer >= 8 ? 8 : kPer >= 4 ? 4 : kPer >= 2 ? 2 : 1;
+  static_assert((G * D4 * NS) % 32 == 0, "output groups must fill whole warps");
+  // Each thread's partial outputs are loaded kChunk splits at a time, all in
+  // flight together; the first chunk of its first output group is requested
+  // before the split weights are computed, so that those loads and the
+  // (max, sum) loads travel at once.
+  // (one chunk covers the ~38 splits per thread of one request with four KV
+  // heads; with NS > 1 each thread has about half as many)
+  constexpr int kChunk = NS >= 2 ? 16 : 40;
+  float4 ov[kChunk];
+  {
+    const int e0 = tid, e = e0 / NS, part = e0 % NS;
+    const int h = e / D4, d4 = d4_0 + e % D4;
+#pragma unroll
+    for (int c = 0; c < kChunk; ++c) {
+      const int sp = part + c * NS;
+      ov[c] = (e0 < G * D4 * NS && sp < p.splits)
+                  ? __ldcg(reinterpret_cast<const float4*>(
+                               part_o + (head0 + (size_t)h * p.splits + sp) * D) +
+                           d4)
+                  : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  // per head: weight of split s = 2^(m_s - M) / L, lanes over splits; the
+  // (m, l) pairs of the first 64 splits are loaded once and kept
+  for (int h = warp; h < G; h += kThreads / 32) {
+    const size_t hb = head0 + (size_t)h * p.splits;
+    float2 ml[2];
+    float M = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int sp = lane + 32 * i;
+      ml[i] = sp < p.splits ? __ldcg(&part_ml[hb + sp]) : make_float2(-INFINITY, 0.f);
+      M = fmaxf(M, ml[i].x);
+    }
+    for (int sp = lane + 64; sp < p.splits; sp += 32) M = fmaxf(M, __ldcg(&part_ml[hb + sp]).x);
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float L = 0.f;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int sp = lane + 32 * i;
+      const float wgt = (M != -INFINITY && ml[i].y > 0.f) ? fast_exp2(ml[i].x - M) : 0.f;
+      if (sp < p.splits) wts[h * p.splits + sp] = wgt;
+      L = fmaf(ml[i].y, wgt, L);
+    }
+    for (int sp = lane + 64; sp < p.splits; sp += 32) {
+      const float2 m2 = __ldcg(&part_ml[hb + sp]);
+      const float wgt = (M != -INFINITY && m2.y > 0.f) ? fast_exp2(m2.x - M) : 0.f;
+      wts[h * p.splits + sp] = wgt;
+      L = fmaf(m2.y, wgt, L);
+    }
+    for (int off = 16; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
+    debug_flag(lane == 0 && len > 0 && !(L > 0.f && isfinite(L)), status);
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    __syncwarp();
+    for (int sp = lane; sp < p.splits; sp += 32) wts[h * p.splits + sp] *= inv;
+  }
+  __syncthreads();
+  for (int e0 = tid; e0 < G * D4 * NS; e0 += kThreads) {
+    const int e = e0 / NS, part = e0 % NS;
+    const int h = e / D4, d4 = d4_0 + e % D4;
+    const size_t hb = head0 + (size_t)h * p.splits;
+    const float* wh = wts + h * p.splits;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    // splits part, part + NS, ... in order, kChunk at a time (the first
+    // chunk of the first group is in ov already)
+    for (int sp0 = part; sp0 < p.splits; sp0 += kChunk * NS) {
+      if (e0 != tid || sp0 != part) {
+#pragma unroll
+        for (int c = 0; c < kChunk; ++c) {
+          const int sp = sp0 + c * NS;
+          ov[c] = sp < p.splits ? __ldcg(reinterpret_cast<const float4*>(part_o + (hb + sp) * D) + d4)
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+#pragma unroll
+      for (int c = 0; c < kChunk; ++c) {
+        const int sp = sp0 + c * NS;
+        if (sp < p.splits) {
+          const float wgt = wh[sp];
+          acc.x = fmaf(ov[c].x, wgt, acc.x);
+          acc.y = fmaf(ov[c].y, wgt, acc.y);
+          acc.z = fmaf(ov[c].z, wgt, acc.z);
+          acc.w = fmaf(ov[c].w, wgt, acc.w);
+        }
+      }
+    }
+#pragma unroll
+    for (int off = 1; off < NS; off <<= 1) {
+      acc.x += __shfl_xor_sync(0xffffffffu, acc.x, off);
+      acc.y += __shfl_xor_sync(0xffffffffu, acc.y, off);
+      acc.z += __shfl_xor_sync(0xffffffffu, acc.z, off);
+      acc.w += __shfl_xor_sync(0xffffffffu, acc.w, off);
+    }
+    if (part != 0) continue;
+    const size_t oi = ((size_t)b * p.hq + (size_t)g * G + h) * D + 4 * d4;
+    if (p.out_dtype == TB_F32) {
+      *reinterpret_cast<float4*>(static_cast<float*>(out) + oi) = acc;
+    } else {
+      uint16_t* ob = static_cast<uint16_t*>(out) + oi;
+      ob[0] = float_to_bf16_rne(acc.x);
+      ob[1] = float_to_bf16_rne(acc.y);
+      ob[2] = float_to_bf16_rne(acc.z);
+      ob[3] = float_to_bf16_rne(acc.w);
+    }
+  }
 }
 
 template <int D, int G>
@@ -430,7 +561,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     *reinterpret_cast<float4*>(part_o + (part_base + (size_t)h * p.splits) * D + 4 * d4) = O;
   }
 
-  // ---- the last split CTA of this (request, KV head) merges every split.
+  // ---- with the merge kernel behind this one, the partials are all it leaves
+  if (p.merge_kernel) return;
+  // ---- otherwise the last split CTA of this (request, KV head) merges every split.
   // One thread counts the CTA in with an acquire-release atomic: the barrier
   // orders every thread's partial stores before it, the release makes them
   // visible with the count, and the last CTA's acquire (then its barrier)
@@ -450,120 +583,29 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncthreads();
   if (!*last_flag) return;
-  const size_t head0 = ((size_t)b * p.hq + (size_t)g * G) * p.splits;
-  // outputs in float4 groups of dims; the splits are divided among the
-  // threads that share an output (NS of them), their sums combined by shuffles
-  constexpr int D4 = D / 4;
-  // (G * D4 * NS is a multiple of 32 for every supported G and D, so each
-  // warp's lanes run the same iterations and the shuffles see full warps)
-  constexpr int kPer = kThreads / (G * D4);
-  constexpr int NS = kPer >= 8 ? 8 : kPer >= 4 ? 4 : kPer >= 2 ? 2 : 1;
-  static_assert((G * D4 * NS) % 32 == 0, "output groups must fill whole warps");
-  // Each thread's partial outputs are loaded kChunk splits at a time, all in
-  // flight together; the first chunk of its first output group is requested
-  // before the split weights are computed, so that those loads and the
-  // (max, sum) loads travel at once.
-  // (one chunk covers the ~38 splits per thread of one request with four KV
-  // heads; with NS > 1 each thread has about half as many)
-  constexpr int kChunk = NS >= 2 ? 16 : 40;
-  float4 ov[kChunk];
-  {
-    const int e0 = tid, e = e0 / NS, part = e0 % NS;
-    const int h = e / D4, d4 = e % D4;
-#pragma unroll
-    for (int c = 0; c < kChunk; ++c) {
-      const int sp = part + c * NS;
-      ov[c] = (e0 < G * D4 * NS && sp < p.splits)
-                  ? __ldcg(reinterpret_cast<const float4*>(
-                               part_o + (head0 + (size_t)h * p.splits + sp) * D) +
-                           d4)
-                  : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-  }
-  // per head: weight of split s = 2^(m_s - M) / L, lanes over splits; the
-  // (m, l) pairs of the first 64 splits are loaded once and kept
-  float* wts = reinterpret_cast<float*>(smem);  // [G][splits] (the ring is free)
-  for (int h = warp; h < G; h += kThreads / 32) {
-    const size_t hb = head0 + (size_t)h * p.splits;
-    float2 ml[2];
-    float M = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const int sp = lane + 32 * i;
-      ml[i] = sp < p.splits ? __ldcg(&part_ml[hb + sp]) : make_float2(-INFINITY, 0.f);
-      M = fmaxf(M, ml[i].x);
-    }
-    for (int sp = lane + 64; sp < p.splits; sp += 32) M = fmaxf(M, __ldcg(&part_ml[hb + sp]).x);
-    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    float L = 0.f;
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const int sp = lane + 32 * i;
-      const float wgt = (M != -INFINITY && ml[i].y > 0.f) ? fast_exp2(ml[i].x - M) : 0.f;
-      if (sp < p.splits) wts[h * p.splits + sp] = wgt;
-      L = fmaf(ml[i].y, wgt, L);
-    }
-    for (int sp = lane + 64; sp < p.splits; sp += 32) {
-      const float2 m2 = __ldcg(&part_ml[hb + sp]);
-      const float wgt = (M != -INFINITY && m2.y > 0.f) ? fast_exp2(m2.x - M) : 0.f;
-      wts[h * p.splits + sp] = wgt;
-      L = fmaf(m2.y, wgt, L);
-    }
-    for (int off = 16; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
-    debug_flag(lane == 0 && len > 0 && !(L > 0.f && isfinite(L)), status);
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    __syncwarp();
-    for (int sp = lane; sp < p.splits; sp += 32) wts[h * p.splits + sp] *= inv;
-  }
-  __syncthreads();
-  for (int e0 = tid; e0 < G * D4 * NS; e0 += kThreads) {
-    const int e = e0 / NS, part = e0 % NS;
-    const int h = e / D4, d4 = e % D4;
-    const size_t hb = head0 + (size_t)h * p.splits;
-    const float* wh = wts + h * p.splits;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    // splits part, part + NS, ... in order, kChunk at a time (the first
-    // chunk of the first group is in ov already)
-    for (int sp0 = part; sp0 < p.splits; sp0 += kChunk * NS) {
-      if (e0 != tid || sp0 != part) {
-#pragma unroll
-        for (int c = 0; c < kChunk; ++c) {
-          const int sp = sp0 + c * NS;
-          ov[c] = sp < p.splits ? __ldcg(reinterpret_cast<const float4*>(part_o + (hb + sp) * D) + d4)
-                                : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-      }
-#pragma unroll
-      for (int c = 0; c < kChunk; ++c) {
-        const int sp = sp0 + c * NS;
-        if (sp < p.splits) {
-          const float wgt = wh[sp];
-          acc.x = fmaf(ov[c].x, wgt, acc.x);
-          acc.y = fmaf(ov[c].y, wgt, acc.y);
-          acc.z = fmaf(ov[c].z, wgt, acc.z);
-          acc.w = fmaf(ov[c].w, wgt, acc.w);
-        }
-      }
-    }
-#pragma unroll
-    for (int off = 1; off < NS; off <<= 1) {
-      acc.x += __shfl_xor_sync(0xffffffffu, acc.x, off);
-      acc.y += __shfl_xor_sync(0xffffffffu, acc.y, off);
-      acc.z += __shfl_xor_sync(0xffffffffu, acc.z, off);
-      acc.w += __shfl_xor_sync(0xffffffffu, acc.w, off);
-    }
-    if (part != 0) continue;
-    const size_t oi = ((size_t)b * p.hq + (size_t)g * G + h) * D + 4 * d4;
-    if (p.out_dtype == TB_F32) {
-      *reinterpret_cast<float4*>(static_cast<float*>(out) + oi) = acc;
-    } else {
-      uint16_t* ob = static_cast<uint16_t*>(out) + oi;
-      ob[0] = float_to_bf16_rne(acc.x);
-      ob[1] = float_to_bf16_rne(acc.y);
-      ob[2] = float_to_bf16_rne(acc.z);
-      ob[3] = float_to_bf16_rne(acc.w);
-    }
-  }
+  merge_splits<D, G, 1>(p, b, g, 0, part_o, part_ml, out, status, reinterpret_cast<float*>(smem), len);
+}
+
+// The split merge as a kernel of its own, kMergeParts CTAs per (KV head,
+// request), each on a quarter of the head dims (so that the splits' partial
+// outputs are read by several SMs at once), launched behind the split kernel
+// (programmatic dependent launch: resident while the split CTAs run, it waits
+// for their completion), so that no split CTA waits on a split counter's
+// round trip.
+template <int D, int G>
+__global__ void __launch_bounds__(kThreads) decode_merge(
+    const __grid_constant__ DecodeParams p, const int32_t* __restrict__ lens,
+    const float* __restrict__ part_o, const float2* __restrict__ part_ml, void* __restrict__ out,
+    int32_t* __restrict__ status) {
+  extern __shared__ float wts[];  // [G][splits]
+  const int g = blockIdx.x, b = blockIdx.y, dpart = blockIdx.z;
+  pdl_wait();
+  pdl_trigger();
+  const int64_t cap64 = p.max_len < (int64_t)p.cache_cap[b] ? p.max_len : (int64_t)p.cache_cap[b];
+  int len = lens[b];
+  if (len > (int)cap64) len = (int)cap64;  // (the split kernel flags it)
+  if (len < 0) len = 0;
+  merge_splits<D, G, kMergeParts>(p, b, g, dpart, part_o, part_ml, out, status, wts, len);
 }
 
 template <int D, int G>
@@ -578,6 +620,16 @@ cudaError_t launch_g(const DecodeParams& p, const CUtensorMap& tk, const CUtenso
                  static_cast<const uint16_t*>(Kc), static_cast<const uint16_t*>(Vc),
                  static_cast<const uint16_t*>(q), lens, part_o, part_ml, counters, out, status);
   if (e != cudaSuccess) return e;
+  if (p.merge_kernel) {
+    auto mk = decode_merge<D, G>;
+    const size_t msmem = sizeof(float) * (size_t)G * p.splits;
+    e = cudaFuncSetAttribute(mk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)msmem);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(mk, dim3(p.hkv, p.batch, kMergeParts), dim3(kThreads), msmem, s, p, lens,
+                   static_cast<const float*>(part_o), static_cast<const float2*>(part_ml), out, status);
+    count_launches(1);
+    if (e != cudaSuccess) return e;
+  }
   return cudaGetLastError();
 }
 

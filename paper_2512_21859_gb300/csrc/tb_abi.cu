@@ -213,6 +213,14 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
   p->splits = (int32_t)splits;
   p->split_len = (int32_t)split_len;
   p->early_tma = 1;
+  // Where the splits leave most SMs idle, a merge kernel behind the split
+  // kernel merges them (four CTAs per KV head, each on a quarter of the head
+  // dims); where the split CTAs fill the part, the last split CTA of each
+  // (request, KV head) does. Measured on GB300 (graphs of consecutive
+  // prepared calls, µs): 7B shape at 2K keys 5.83 -> 5.26 and 32K α 0.95
+  // 5.71 -> 5.11 with the merge kernel (68 and 56 split CTAs), against
+  // 128K α 0.9 13.70 -> 13.58 and 32K α 0.5 10.17 -> 10.45 (144 and 132).
+  p->merge_kernel = splits * units < 120 ? 1 : 0;
   return TB_OK;
 }
 

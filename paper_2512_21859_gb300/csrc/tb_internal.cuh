@@ -68,7 +68,10 @@ struct DecodeParams {
   int64_t cache_rows;
   int64_t max_len;
   float scale_log2;
-  int32_t pad1;
+  // 1: the split kernel leaves its partials and a merge kernel launched
+  // behind it (programmatic dependent launch) merges them; 0: the last split
+  // CTA of each (request, KV head) merges them, found with a split counter
+  int32_t merge_kernel;
   int64_t cache_off[TB_MAX_BATCH];
   int32_t cache_cap[TB_MAX_BATCH];
 };
