@@ -213,14 +213,15 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
   p->splits = (int32_t)splits;
   p->split_len = (int32_t)split_len;
   p->early_tma = 1;
-  // Where the splits leave most SMs idle, a merge kernel behind the split
-  // kernel merges them (four CTAs per KV head, each on a quarter of the head
-  // dims); where the split CTAs fill the part, the last split CTA of each
-  // (request, KV head) does. Measured on GB300 (graphs of consecutive
-  // prepared calls, µs): 7B shape at 2K keys 5.83 -> 5.26 and 32K α 0.95
-  // 5.71 -> 5.11 with the merge kernel (68 and 56 split CTAs), against
-  // 128K α 0.9 13.70 -> 13.58 and 32K α 0.5 10.17 -> 10.45 (144 and 132).
-  p->merge_kernel = splits * units < 120 ? 1 : 0;
+  // When every split is a single 128-key tile (short caches), a merge kernel
+  // behind the split kernel merges the splits (four CTAs per KV head, each
+  // on a quarter of the head dims); with longer splits the last split CTA of
+  // each (request, KV head) does. Measured on GB300 (graphs of consecutive
+  // prepared calls, µs, last CTA -> merge kernel): one-tile splits: 7B shape
+  // at 2K keys 5.81 -> 5.23, at 4K 6.42 -> 5.92, 32K α 0.95 5.73 -> 5.15;
+  // longer splits: 7B shape at 8K 7.65 -> 7.81, 32K α 0.75 7.64 -> 7.81,
+  // α 0.5 10.23 -> 10.45, 128K α 0.75 25.69 -> 25.92, α 0.9 13.75 -> 13.59.
+  p->merge_kernel = split_len <= 128 ? 1 : 0;
   return TB_OK;
 }
 
