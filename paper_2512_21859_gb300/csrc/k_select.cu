@@ -172,8 +172,12 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
 constexpr int kCsThreads = 1024;
 constexpr int kCsWarps = kCsThreads / 32;
 
+// 32-key chunks of one warp's run in the compaction (runs of up to 512 keys)
+constexpr int kRunChunks = kClusterSliceMax / kCsThreads;
+
 struct ClusterSelectShared {
   unsigned hist[2][256];
+  uint2 masks[kCsWarps][kRunChunks];  // per chunk: ballots of (key > tau, key == tau)
   unsigned total[256];
   int wgt[kCsWarps], weq[kCsWarps];
   int cta_cnt[2];  // this CTA's (greater, equal) counts, read by the cluster
@@ -338,10 +342,11 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
         }
       }
       cluster.sync();
-      for (int t = tid; t < 256; t += kCsThreads) {
-        unsigned sum = 0;
-        for (int r = 0; r < cs; ++r) sum += cluster.map_shared_rank(h, r)[t];
-        sh.total[t] = sum;
+      if (tid < 256) {
+        unsigned v[8];
+#pragma unroll
+        for (int r = 0; r < 8; ++r) v[r] = r < cs ? cluster.map_shared_rank(h, r)[tid] : 0u;
+        sh.total[tid] = ((v[0] + v[1]) + (v[2] + v[3])) + ((v[4] + v[5]) + (v[6] + v[7]));
       }
       __syncthreads();
       if (warp == 0) {
@@ -393,8 +398,12 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int i = b0 + 32 * q + lane;
-        gt_w += __popc(__ballot_sync(0xffffffffu, i < whi && kv[q] > tau));
-        eq_w += __popc(__ballot_sync(0xffffffffu, i < whi && kv[q] == tau));
+        const unsigned gm = __ballot_sync(0xffffffffu, i < whi && kv[q] > tau);
+        const unsigned em = __ballot_sync(0xffffffffu, i < whi && kv[q] == tau);
+        // the chunk's ballots, for the emission pass
+        if (lane == q && b0 + 32 * q < whi) sh.masks[warp][(b0 - wlo) / 32 + q] = make_uint2(gm, em);
+        gt_w += __popc(gm);
+        eq_w += __popc(em);
       }
     }
   }
@@ -436,28 +445,23 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
     eqbase += sh.weq[w];
   }
   if (k > 0) {
+    // emission from the count pass's ballots: per 32-key chunk, the keys
+    // above tau and the first ties until `need` of them are kept
     const unsigned lt = (1u << lane) - 1u;
-    for (int b0 = wlo; b0 < whi; b0 += 128) {
-      unsigned kv[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int i = b0 + 32 * q + lane;
-        kv[q] = i < whi ? keys[i] : 0u;
-      }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int i = b0 + 32 * q + lane;
-        const bool gt = i < whi && kv[q] > tau;
-        const bool eq = i < whi && kv[q] == tau;
-        const unsigned em = __ballot_sync(0xffffffffu, eq);
-        const bool sel = gt || (eq && eqbase + __popc(em & lt) < need);
-        const unsigned sm = __ballot_sync(0xffffffffu, sel);
-        const int pos = selbase + __popc(sm & lt);
-        if (sel && pos < k) out[pos] = lo + i;
-        debug_flag(sel && pos >= k, status);
-        selbase += __popc(sm);
-        eqbase += __popc(em);
-      }
+    const int nch = (whi - wlo + 31) / 32;
+    for (int c = 0; c < nch; ++c) {
+      const uint2 m = sh.masks[warp][c];
+      const int room = need - eqbase;  // ties still to keep
+      unsigned tie = room > 0 ? m.y : 0u;
+      if (room > 0 && __popc(tie) > room)  // the chunk where the ties run out
+        tie = __ballot_sync(0xffffffffu, ((m.y >> lane) & 1u) && __popc(m.y & lt) < room);
+      const unsigned sm = m.x | tie;
+      const int pos = selbase + __popc(sm & lt);
+      const bool sel = (sm >> lane) & 1u;
+      if (sel && pos < k) out[pos] = lo + wlo + 32 * c + lane;
+      debug_flag(sel && pos >= k, status);
+      selbase += __popc(sm);
+      eqbase += __popc(m.y);
     }
   }
   // the cluster's last warp ends on the total: exactly k positions kept
