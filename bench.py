@@ -313,8 +313,17 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
     ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
                           cache_offset=desc.out_offset, cache_cap=desc.out_cap,
                           cache_rows=desc.out_rows, max_len=max(lens_h), flags=tb.TB_DECODE_EARLY_CACHE_READ)
+    # the step's decode runs beside the select (TB_DECODE_CONCURRENT) on the
+    # SMs the select leaves free: its own descriptor and prepared workspaces
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    step_ctas = max(1, sms - tb.tb_select_ctas(desc))
+    sddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
+                           cache_offset=desc.out_offset, cache_cap=desc.out_cap, cache_rows=desc.out_rows,
+                           max_len=max(lens_h), flags=tb.TB_DECODE_EARLY_CACHE_READ | tb.TB_DECODE_CONCURRENT,
+                           max_ctas=step_ctas)
     ews = tb.tb_evict_workspace_size(desc)
     dws = tb.tb_decode_workspace_size(ddesc)
+    sdws = tb.tb_decode_workspace_size(sddesc)
     step_in = inputs.make_decode_step(wl, rank, 1, B)
     q_dec = to_device(torch, wl, step_in["q"], dev)
     kn, vn = to_device(torch, wl, step_in["k_new"], dev), to_device(torch, wl, step_in["v_new"], dev)
@@ -332,6 +341,8 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
         d["ews"] = torch.empty(ews, dtype=torch.uint8, device=dev)
         d["dws"] = torch.empty(dws, dtype=torch.uint8, device=dev)
         tb.tb_decode_workspace_prepare(ddesc, d["dws"], stream=stream)
+        d["sdws"] = torch.empty(sdws, dtype=torch.uint8, device=dev)
+        tb.tb_decode_workspace_prepare(sddesc, d["sdws"], stream=stream)
         d["out"] = torch.empty((B, wl.hq, wl.head_dim), dtype=torch.float32, device=dev)
         bufs.append(d)
     lens = torch.tensor(lens_h, dtype=torch.int32, device=dev)
@@ -339,6 +350,8 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
     def stage_call(name, d, st):
         if name == "decode_attn":
             tb.tb_decode_attn_prepared(ddesc, q_dec, d["Kc"], d["Vc"], lens, d["out"], d["dws"], stream=st)
+        elif name == "decode_beside_select":
+            tb.tb_decode_attn_prepared(sddesc, q_dec, d["Kc"], d["Vc"], lens, d["out"], d["sdws"], stream=st)
         elif name == "window_scores":
             tb.tb_window_scores(desc, d["q_win"], d["K"], d["scores"], d["ews"], stream=st)
         elif name == "select_topk":
@@ -365,12 +378,15 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
         dec_bufs.append(d)
     torch.cuda.synchronize(dev)
     return {"desc": desc, "ddesc": ddesc, "bufs": bufs, "dec_bufs": dec_bufs, "R": R, "ab": ab,
-            "stage_call": stage_call, "step_in": step_in, "ews": ews, "dws": dws}
+            "stage_call": stage_call, "step_in": step_in, "ews": ews, "dws": dws, "step_ctas": step_ctas}
 
 
 def check_decode_status(tb, stream, S):
     for d in S["dec_bufs"]:
         st, raw = tb.tb_read_status(d["dws"], stream=stream)
+        assert st == tb.TB_OK, raw
+    for d in S["bufs"]:
+        st, raw = tb.tb_read_status(d["sdws"], stream=stream)
         assert st == tb.TB_OK, raw
 
 
@@ -418,18 +434,21 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     ab, R, desc, ddesc = S["ab"], S["R"], S["desc"], S["ddesc"]
     stage_call = S["stage_call"]
     layers = S["bufs"]
+    step_ctas = S["step_ctas"]
 
-    # each layer buffer's step captured into a CUDA graph of the four calls
-    # on one stream. Default order: window scoring, select, decode, gather.
-    # The select runs one cluster per KV head and leaves most SMs idle; the
-    # decode, a programmatic dependent launch behind it, gets its CTAs
-    # resident there during the select and requests its first tiles before
-    # its dependency wait (its early-read assertion holds: the select writes
-    # only indices). That decode attends over the compacted cache of the
+    # each layer buffer's step captured into a CUDA graph of the four calls.
+    # Default: window scoring, then the select; the decode, the select's
+    # programmatic dependent with TB_DECODE_CONCURRENT and a CTA budget of
+    # the SMs the select leaves free, runs beside the select (the select
+    # runs one cluster per KV head and is bound by its phases' latency, the
+    # decode by HBM); the gather follows the select on a second stream (an
+    # event recorded after the select), and the step ends when both
+    # branches have. The decode attends over the compacted cache of the
     # previous buffer of the rotation (the previous step's eviction output),
-    # never over the cache this step's gather writes. --serial-step: the
-    # decode first, then the eviction, over the buffer's own cache.
+    # which nothing in the step writes. --serial-step: the decode first,
+    # then the eviction, over the buffer's own cache, on one stream.
     cap = torch.cuda.Stream(dev)
+    side = torch.cuda.Stream(dev)
     step_graphs = []
     kernels_per_step = None
     for i, d in enumerate(layers):
@@ -442,8 +461,10 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             else:
                 stage_call("window_scores", d, cap)
                 stage_call("select_topk", d, cap)
-                stage_call("decode_attn", layers[(i + L - 1) % L], cap)
-                stage_call("gather_kv", d, cap)
+                side.wait_stream(cap)
+                stage_call("decode_beside_select", layers[(i + L - 1) % L], cap)
+                stage_call("gather_kv", d, side)
+                cap.wait_stream(side)
         kernels_per_step = tb.tb_launch_counter() - c0
         step_graphs.append(g)
     torch.cuda.synchronize(dev)
@@ -526,12 +547,15 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                 L, W["layer_bytes"] / 1e6),
             "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
             "decode_call": "tb_decode_attn_prepared with TB_DECODE_EARLY_CACHE_READ (workspace prepared once; "
-                           "no per-call clearing kernel; first tiles requested before the preceding kernel ends)",
+                           "no per-call clearing kernel; first tiles requested before the preceding kernel ends); "
+                           "in the step also with TB_DECODE_CONCURRENT and max_ctas (no dependency wait: it "
+                           "runs beside the select)",
             "launch": "each step is one CUDA-graph replay of the four C-ABI calls" + (
                 ": decode_attn, window_scores, select_topk, gather_kv" if args.serial_step else
-                " in the order window_scores, select_topk, decode_attn, gather_kv: the decode's CTAs "
-                "start during the select (programmatic dependent launch) on the SMs it leaves free and "
-                "attend over the previous rotation buffer's compacted cache"),
+                ": window_scores, select_topk, then the decode (TB_DECODE_CONCURRENT, the select's "
+                "programmatic dependent, max_ctas = SMs - tb_select_ctas = %d) beside the select, over "
+                "the previous rotation buffer's compacted cache, and gather_kv after the select on a "
+                "second stream" % step_ctas),
             "stage_timing": stage_timing,
             "parallelism": "replicas" if world > 1 else "single GPU"},
         "us_per_layer": {"evict": round(evict_us, 2), "decode": round(1e3 * stage_ms["decode_attn"], 2),

@@ -75,7 +75,8 @@ typedef enum { TB_F32 = 0, TB_BF16 = 1 } tb_dtype;
 /* Static description of a status code; never NULL. */
 const char *tb_status_string(int32_t status);
 
-/* Version of this ABI (major * 100 + minor): 101 (tb_decode_desc.flags). */
+/* Version of this ABI (major * 100 + minor): 102 (tb_decode_desc.max_ctas,
+ * TB_DECODE_CONCURRENT, tb_select_ctas). */
 int32_t tb_abi_version(void);
 
 /* Text of the last CUDA error this thread saw inside the library (the
@@ -192,6 +193,15 @@ tb_status tb_select_topk(const tb_evict_desc *desc, const float *scores,
                          size_t workspace_bytes, tb_stream_t stream);
 
 /*
+ * Number of CTAs the select of tb_select_topk (and of tb_score_evict) runs
+ * for this descriptor, each on an SM of its own (a thread-block cluster of up
+ * to eight per request and KV head; one per request and KV head on the
+ * fallback path). A decode with TB_DECODE_CONCURRENT launched behind the
+ * select fits beside it with max_ctas = SM count - this. No device work.
+ */
+tb_status tb_select_ctas(const tb_evict_desc *desc, int32_t *ctas);
+
+/*
  * Step 6: Kc[g][out_offset[b] + r] = K[g][kv_offset[b] + idx[g][.. + r]]
  * and the same for V, for r < R_b (bit copies). idx entries must lie in
  * [0, N_b); an entry outside it is skipped and its row left untouched.
@@ -221,6 +231,20 @@ tb_status tb_score_evict(const tb_evict_desc *desc, const void *q_win,
  * tb_decode_attn and tb_decode_attn_noalloc, whose own clearing kernel
  * already lets them do so. */
 #define TB_DECODE_EARLY_CACHE_READ 1
+/* The caller asserts that the work enqueued on the stream just before a
+ * tb_decode_attn_prepared call writes nothing the call reads (q, Kc, Vc,
+ * lens) and touches neither out nor the workspace, and that everything the
+ * call reads was complete before that work was launched. The decode kernel
+ * then does not wait for that work at all: launched behind a kernel that
+ * lets its dependents start early (the library's select and gather kernels
+ * do, right after their own dependency wait), it runs beside it on the SMs
+ * that kernel leaves free (size it with max_ctas, e.g. the SM count minus
+ * tb_select_ctas). The call's completion then says nothing about that
+ * work's: whatever needs the preceding kernel's results must be ordered
+ * after it by an event recorded before this call. Implies
+ * TB_DECODE_EARLY_CACHE_READ. No effect on tb_decode_attn and
+ * tb_decode_attn_noalloc (their clearing kernel comes first). */
+#define TB_DECODE_CONCURRENT 2
 
 /* Shape of one batched decode step. */
 typedef struct {
@@ -235,6 +259,11 @@ typedef struct {
   int64_t cache_rows;          /* rows per KV head of Kc and Vc */
   int64_t max_len;             /* upper bound of lens[b], >= 1 */
   int32_t flags;               /* TB_DECODE_* bits; any other bit is an error */
+  int32_t max_ctas;            /* 0: about one CTA per SM of a 152-SM GB300
+                                  (the keys of each (request, KV head) split
+                                  that many ways); > 0: at most max(this,
+                                  batch * hkv) CTAs, in fewer, longer splits;
+                                  < 0 is an error */
 } tb_decode_desc;
 
 /* Bytes of device workspace tb_decode_attn needs for this descriptor. */

@@ -21,8 +21,9 @@ __all__ = [
     "TbError", "EvictDesc", "DecodeDesc", "library_path", "load",
     "tb_status_string", "tb_abi_version", "tb_last_error_detail", "tb_launch_counter",
     "tb_retained_count", "tb_retained_count_ex", "TB_EVICT_BUDGET_INCLUDES_WINDOW",
-    "TB_EVICT_AVG_POOL", "TB_DECODE_EARLY_CACHE_READ", "tb_evict_layout", "tb_evict_workspace_size",
-    "tb_window_scores", "tb_window_scores_lse", "tb_select_topk", "tb_gather_kv", "tb_score_evict",
+    "TB_EVICT_AVG_POOL", "TB_DECODE_EARLY_CACHE_READ", "TB_DECODE_CONCURRENT", "tb_evict_layout",
+    "tb_evict_workspace_size", "tb_window_scores", "tb_window_scores_lse", "tb_select_topk",
+    "tb_select_ctas", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
     "tb_decode_attn_noalloc", "tb_decode_noalloc_status", "TB_NOALLOC_SCRATCH_BYTES", "tb_diag_bounded_wait",
     "tb_decode_workspace_prepare", "tb_decode_attn_prepared",
@@ -32,7 +33,7 @@ __all__ = [
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
 TB_F32, TB_BF16 = 0, 1
 TB_EVICT_BUDGET_INCLUDES_WINDOW, TB_EVICT_AVG_POOL = 1, 2
-TB_DECODE_EARLY_CACHE_READ = 1
+TB_DECODE_EARLY_CACHE_READ, TB_DECODE_CONCURRENT = 1, 2
 TB_MAX_BATCH = 64
 TB_NOALLOC_SCRATCH_BYTES = 4 << 20
 
@@ -55,7 +56,7 @@ class _DecodeDescC(ctypes.Structure):
         ("batch", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
         ("head_dim", ctypes.c_int32), ("dtype", ctypes.c_int32), ("out_dtype", ctypes.c_int32),
         ("cache_offset", _I64P), ("cache_cap", _I64P), ("cache_rows", ctypes.c_int64),
-        ("max_len", ctypes.c_int64), ("flags", ctypes.c_int32),
+        ("max_len", ctypes.c_int64), ("flags", ctypes.c_int32), ("max_ctas", ctypes.c_int32),
     ]
 
 
@@ -106,6 +107,7 @@ def load():
         "tb_window_scores": (I, [P, P, P, P, P, SZ, P]),
         "tb_window_scores_lse": (I, [P, P, P, P, P, P, SZ, P]),
         "tb_select_topk": (I, [P, P, P, P, P, SZ, P]),
+        "tb_select_ctas": (I, [P, ctypes.POINTER(I)]),
         "tb_gather_kv": (I, [P, P, P, P, P, P, P]),
         "tb_score_evict": (I, [P, P, P, P, P, P, P, P, P, SZ, P]),
         "tb_decode_workspace_size": (I, [P, ctypes.POINTER(SZ)]),
@@ -221,14 +223,16 @@ class DecodeDesc:
     """tb_decode_desc plus its host arrays."""
 
     def __init__(self, *, hq: int, hkv: int, head_dim: int, dtype: int, cache_offset,
-                 cache_cap, cache_rows: int, max_len: int, out_dtype: int = TB_F32, flags: int = 0):
+                 cache_cap, cache_rows: int, max_len: int, out_dtype: int = TB_F32, flags: int = 0,
+                 max_ctas: int = 0):
         self.cache_offset = np.ascontiguousarray(cache_offset, dtype=np.int64)
         self.cache_cap = np.ascontiguousarray(cache_cap, dtype=np.int64)
         self.flags = int(flags)
+        self.max_ctas = int(max_ctas)
         self.c = _DecodeDescC(
             int(self.cache_offset.shape[0]), hq, hkv, head_dim, dtype, out_dtype,
             self.cache_offset.ctypes.data_as(_I64P), self.cache_cap.ctypes.data_as(_I64P),
-            int(cache_rows), int(max_len), self.flags)
+            int(cache_rows), int(max_len), self.flags, self.max_ctas)
         self.hq, self.hkv, self.head_dim, self.dtype, self.out_dtype = hq, hkv, head_dim, dtype, out_dtype
         self.cache_rows, self.max_len = int(cache_rows), int(max_len)
 
@@ -313,6 +317,13 @@ def tb_select_topk(desc: EvictDesc, scores, idx, pooled, workspace, workspace_by
     w, wb = _ws(workspace, workspace_bytes)
     _check(load().tb_select_topk(desc.ref(), _ptr(scores), _ptr(idx), _ptr(pooled), w, wb,
                                  _stream(stream)), "tb_select_topk")
+
+
+def tb_select_ctas(desc: EvictDesc) -> int:
+    """CTAs (one per SM) the select of this descriptor runs."""
+    n = ctypes.c_int32()
+    _check(load().tb_select_ctas(desc.ref(), ctypes.byref(n)), "tb_select_ctas")
+    return int(n.value)
 
 
 def tb_gather_kv(desc: EvictDesc, idx, K, V, Kc, Vc, stream=None):

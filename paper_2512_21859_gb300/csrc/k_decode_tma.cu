@@ -290,9 +290,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   // the cache rows cannot be written by the clearing kernel. Mode 2: the
   // caller asserts the same of the work before this kernel for every row
   // below lens[b] - 1; that last row (appended by the decode loop, possibly
-  // by the preceding kernel) is read again after the wait, below. Without it
-  // (a prepared workspace, no assertion) any kernel may precede this one, so
-  // the requests wait for it.
+  // by the preceding kernel) is read again after the wait, below. Mode 3:
+  // the caller asserts that the preceding kernel writes nothing this one
+  // reads and that everything it reads was complete before that kernel was
+  // launched, so there is no wait at all and this kernel runs beside it.
+  // Without either (a prepared workspace, no assertion) any kernel may
+  // precede this one, so the requests wait for it.
   int issued = 0;
   if (tid == 0) {
     tc::tma_prefetch_desc(&tk);
@@ -300,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (p.early_tma)
       for (; issued < kStages && issued < ntiles_c; ++issued) issue(issued);
   }
-  pdl_wait();
+  if (p.early_tma != 3) pdl_wait();
   pdl_trigger();
   if (tid == 0)
     for (; issued < kStages && issued < ntiles_c; ++issued) issue(issued);

@@ -170,7 +170,8 @@ tb_status check_ws(void* ws, size_t bytes, size_t need) {
 tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
   if (!d) return TB_ERR_INVALID_ARG;
   if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->max_len < 1) return TB_ERR_INVALID_ARG;
-  if ((d->flags & ~TB_DECODE_EARLY_CACHE_READ) != 0) return TB_ERR_INVALID_ARG;
+  if ((d->flags & ~(TB_DECODE_EARLY_CACHE_READ | TB_DECODE_CONCURRENT)) != 0 || d->max_ctas < 0)
+    return TB_ERR_INVALID_ARG;
   if (d->batch > TB_MAX_BATCH) return TB_ERR_UNSUPPORTED;
   if (d->hq % d->hkv != 0) return TB_ERR_INVALID_ARG;
   if (d->dtype != TB_F32 && d->dtype != TB_BF16) return TB_ERR_UNSUPPORTED;
@@ -201,10 +202,11 @@ tb_status build_decode(const tb_decode_desc* d, DecodeParams* p) {
     p->cache_cap[b] = (int32_t)d->cache_cap[b];
   }
   // Split the keys so that about one CTA per SM of a 152-SM part runs, in
-  // whole 128-key tiles (each CTA keeps three tiles in flight).
-  const int64_t target = 152;
+  // whole 128-key tiles (each CTA keeps three tiles in flight); with a CTA
+  // budget, as many splits per (request, KV head) as it holds (at least one).
+  // Rounding the split length up to whole tiles only lowers the count.
   const int64_t units = (int64_t)d->batch * d->hkv;
-  int64_t splits = (target + units - 1) / units;
+  int64_t splits = d->max_ctas > 0 ? d->max_ctas / units : (152 + units - 1) / units;
   const int64_t max_splits = (d->max_len + 127) / 128;
   splits = std::max<int64_t>(1, std::min(splits, max_splits));
   int64_t split_len = (d->max_len + splits - 1) / splits;
@@ -340,7 +342,7 @@ const char* tb_status_string(int32_t status) {
   }
 }
 
-int32_t tb_abi_version(void) { return 101; }
+int32_t tb_abi_version(void) { return 102; }
 
 const char* tb_last_error_detail(void) { return g_last_error; }
 
@@ -557,6 +559,16 @@ tb_status tb_select_topk(const tb_evict_desc* desc, const float* scores, int32_t
   return run_select(p, w, scores, idx, pooled, workspace, s);
 }
 
+tb_status tb_select_ctas(const tb_evict_desc* desc, int32_t* ctas) {
+  if (!ctas) return TB_ERR_INVALID_ARG;
+  EvictParams p;
+  const tb_status st = build_evict(desc, &p);
+  if (st != TB_OK) return st;
+  const int per = select_cluster_supported(p) ? select_cluster_size(p) : 1;
+  *ctas = p.batch * p.hkv * per;
+  return TB_OK;
+}
+
 tb_status tb_gather_kv(const tb_evict_desc* desc, const int32_t* idx, const void* K,
                        const void* V, void* Kc, void* Vc, tb_stream_t stream) {
   const NvtxRange range("tb_gather_kv");
@@ -648,8 +660,11 @@ tb_status tb_decode_attn_prepared(const tb_decode_desc* desc, const void* q, con
   // prepared (each call's last split CTA zeroes its counter again), and the
   // status word keeps what earlier calls raised. Any kernel may precede this
   // one, so its first tiles wait for it, unless the caller asserts that the
-  // preceding work writes no cache row below the last appended one
-  p.early_tma = (desc->flags & TB_DECODE_EARLY_CACHE_READ) ? 2 : 0;
+  // preceding work writes no cache row below the last appended one (mode 2),
+  // or that it writes nothing this call reads and needs no wait at all (3)
+  p.early_tma = (desc->flags & TB_DECODE_CONCURRENT)         ? 3
+                : (desc->flags & TB_DECODE_EARLY_CACHE_READ) ? 2
+                                                             : 0;
   return cuda_status(launch_decode(p, q, Kc, Vc, lens, out, at<float>(workspace, w.part_o),
                                    at<float2>(workspace, w.part_ml),
                                    at<int32_t>(workspace, w.counters),

@@ -62,8 +62,10 @@ struct DecodeParams {
   // clearing kernel, so the first K/V tiles may be requested before the
   // dependency wait; 2: the same on the caller's word (prepared workspace
   // with TB_DECODE_EARLY_CACHE_READ) that the work before it writes no cache
-  // row below lens[b] - 1, which is read again after the wait; 0 (prepared
-  // workspaces otherwise): anything may precede it
+  // row below lens[b] - 1, which is read again after the wait; 3
+  // (TB_DECODE_CONCURRENT): no dependency wait at all, the work before it
+  // writes nothing the decode reads; 0 (prepared workspaces otherwise):
+  // anything may precede it
   int32_t early_tma;
   int64_t cache_rows;
   int64_t max_len;

@@ -43,7 +43,7 @@ def test_status_strings_and_version(tb):
     for s in range(6):
         assert tb.tb_status_string(s)
     assert tb.tb_status_string(99) == "unknown status"
-    assert tb.tb_abi_version() == 101
+    assert tb.tb_abi_version() == 102
     assert tb.tb_last_error_detail() == ""
 
 
@@ -152,6 +152,46 @@ def test_decode_workspace(tb):
     assert a > 256 and b >= a
 
 
+def test_decode_cta_budget_shrinks_the_splits(tb):
+    """A CTA budget gives fewer splits, so the split partials (and the
+    workspace) shrink; flags with the concurrency bit are accepted."""
+    full = tb.tb_decode_workspace_size(_ddesc(tb))
+    assert tb.tb_decode_workspace_size(_ddesc(tb, max_ctas=152)) == full
+    prev = full
+    for m in (88, 40, 8, 4, 1):
+        w = tb.tb_decode_workspace_size(_ddesc(tb, max_ctas=m, flags=tb.TB_DECODE_CONCURRENT))
+        assert w <= prev
+        prev = w
+    assert prev < full
+    # a budget below one CTA per (request, KV head) still gives one split each
+    assert tb.tb_decode_workspace_size(_ddesc(tb, max_ctas=1)) == tb.tb_decode_workspace_size(
+        _ddesc(tb, max_ctas=4))
+
+
+@pytest.mark.parametrize("n,w,hkv,batch,want", [
+    (512, 16, 2, 1, 2),              # prefix 496: one CTA per cluster
+    (4096 + 16, 16, 2, 1, 2),        # 4096 prefix keys: still one
+    (4096 + 17, 16, 2, 1, 4),        # one more key: two per cluster
+    (32768, 32, 4, 1, 32),           # 32K prefix: eight per cluster
+    (131072, 64, 8, 1, 64),          # 128K: eight per cluster, eight KV heads
+    (131072, 64, 8, 2, 128),         # two requests
+])
+def test_select_ctas(tb, n, w, hkv, batch, want):
+    d = tb.EvictDesc(hq=4 * hkv, hkv=hkv, head_dim=64, window=w, pool_k=7, dtype=tb.TB_F32,
+                     n=[n] * batch, alpha=[0.5] * batch)
+    assert tb.tb_select_ctas(d) == want
+
+
+def test_select_ctas_fallback_and_errors(tb):
+    # a prefix longer than eight 16K slices runs the one-CTA-per-segment fallback
+    d = tb.EvictDesc(hq=4, hkv=2, head_dim=64, window=16, pool_k=7, dtype=tb.TB_F32,
+                     n=[8 * 16384 + 100], alpha=[0.5])
+    assert tb.tb_select_ctas(d) == 2
+    with pytest.raises(tb.TbError) as e:
+        tb.tb_select_ctas(_desc(tb, hq=5))
+    assert e.value.status == tb.TB_ERR_INVALID_ARG
+
+
 @pytest.mark.parametrize("kw,status", [
     (dict(hq=30), 1),
     (dict(head_dim=80), 2),
@@ -161,7 +201,8 @@ def test_decode_workspace(tb):
     (dict(cache_rows=100), 1),
     (dict(cache_offset=[-4]), 1),
     (dict(hq=132, hkv=4), 2),                   # group of 33 heads at d=128
-    (dict(flags=2), 1),                         # an undefined flag bit
+    (dict(flags=4), 1),                         # an undefined flag bit
+    (dict(max_ctas=-1), 1),                     # a negative CTA budget
 ])
 def test_decode_desc_rejects(tb, kw, status):
     with pytest.raises(tb.TbError) as e:
