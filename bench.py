@@ -307,6 +307,10 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
                         pool_k=wl.pool_k, dtype=tb.TB_BF16 if wl.dtype == "bf16" else tb.TB_F32,
                         n=n, alpha=alpha_vec, kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)),
                         out_cap=lens_h)
+    # the step's gather runs beside the next layer's select (no dependency wait)
+    gdesc = tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, window=wl.window,
+                         pool_k=wl.pool_k, dtype=desc.dtype, n=n, alpha=alpha_vec, kv_offset=lay["kv_offset"],
+                         kv_rows=int(np.sum(n)), out_cap=lens_h, flags=tb.TB_EVICT_GATHER_CONCURRENT)
     score_rows, idx_rows = tb.tb_evict_layout(desc)
     # the step's own K/V row is in place before the decode, and the kernel
     # before each decode writes no row of its cache: the early-read assertion holds
@@ -352,6 +356,8 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
             tb.tb_decode_attn_prepared(ddesc, q_dec, d["Kc"], d["Vc"], lens, d["out"], d["dws"], stream=st)
         elif name == "decode_beside_select":
             tb.tb_decode_attn_prepared(sddesc, q_dec, d["Kc"], d["Vc"], lens, d["out"], d["sdws"], stream=st)
+        elif name == "gather_beside_select":
+            tb.tb_gather_kv(gdesc, d["idx"], d["K"], d["V"], d["Kc"], d["Vc"], stream=st)
         elif name == "window_scores":
             tb.tb_window_scores(desc, d["q_win"], d["K"], d["scores"], d["ews"], stream=st)
         elif name == "select_topk":
@@ -436,19 +442,21 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     layers = S["bufs"]
     step_ctas = S["step_ctas"]
 
-    # each layer buffer's step captured into a CUDA graph of the four calls.
-    # Default: window scoring, then the select; the decode, the select's
-    # programmatic dependent with TB_DECODE_CONCURRENT and a CTA budget of
-    # the SMs the select leaves free, runs beside the select (the select
-    # runs one cluster per KV head and is bound by its phases' latency, the
-    # decode by HBM); the gather follows the select on a second stream (an
-    # event recorded after the select), and the step ends when both
-    # branches have. The decode attends over the compacted cache of the
-    # previous buffer of the rotation (the previous step's eviction output),
-    # which nothing in the step writes. --serial-step: the decode first,
-    # then the eviction, over the buffer's own cache, on one stream.
+    # each layer buffer's step captured into a CUDA graph of the four calls,
+    # pipelined over the layer rotation: step i scores layer i and selects
+    # its rows; beside that select (bound by the latency of its phases on
+    # the SMs its clusters hold) run, without dependency waits, the decode
+    # over layer i-2's compacted cache (TB_DECODE_CONCURRENT, a CTA budget
+    # of the SMs the select leaves free) and the gather of layer i-1 (its
+    # rows selected in step i-1; TB_EVICT_GATHER_CONCURRENT), both bound by
+    # HBM. Nothing in the step writes what another call of it reads: the
+    # gather writes layer i-1's compacted cache, the decode reads layer
+    # i-2's (distinct buffers: at least two in the rotation). Every step
+    # thus does one layer's scoring, select, gather and decode step.
+    # --serial-step: the decode first, then the eviction, over the buffer's
+    # own cache, on one stream.
+    assert L >= 2
     cap = torch.cuda.Stream(dev)
-    side = torch.cuda.Stream(dev)
     step_graphs = []
     kernels_per_step = None
     for i, d in enumerate(layers):
@@ -461,10 +469,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             else:
                 stage_call("window_scores", d, cap)
                 stage_call("select_topk", d, cap)
-                side.wait_stream(cap)
-                stage_call("decode_beside_select", layers[(i + L - 1) % L], cap)
-                stage_call("gather_kv", d, side)
-                cap.wait_stream(side)
+                stage_call("decode_beside_select", layers[(i + L - 2) % L], cap)
+                stage_call("gather_beside_select", layers[(i + L - 1) % L], cap)
         kernels_per_step = tb.tb_launch_counter() - c0
         step_graphs.append(g)
     torch.cuda.synchronize(dev)
@@ -545,17 +551,18 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             "workload": describe(wl, n, a), "alpha": float(a[0]) if len(set(a.tolist())) == 1 else a.tolist(),
             "layers_rotated": L, "l2": "inputs larger than L2: %d rotating layer buffers of %.0f MB" % (
                 L, W["layer_bytes"] / 1e6),
-            "step": "decode_attn (one token) + window_scores + select_topk + gather_kv of one layer",
+            "step": "one layer's window_scores + select_topk + gather_kv + decode_attn (one token); "
+                    "pipelined, the gather and the decode are of the previous layers (see launch)",
             "decode_call": "tb_decode_attn_prepared with TB_DECODE_EARLY_CACHE_READ (workspace prepared once; "
                            "no per-call clearing kernel; first tiles requested before the preceding kernel ends); "
                            "in the step also with TB_DECODE_CONCURRENT and max_ctas (no dependency wait: it "
                            "runs beside the select)",
             "launch": "each step is one CUDA-graph replay of the four C-ABI calls" + (
                 ": decode_attn, window_scores, select_topk, gather_kv" if args.serial_step else
-                ": window_scores, select_topk, then the decode (TB_DECODE_CONCURRENT, the select's "
-                "programmatic dependent, max_ctas = SMs - tb_select_ctas = %d) beside the select, over "
-                "the previous rotation buffer's compacted cache, and gather_kv after the select on a "
-                "second stream" % step_ctas),
+                ", pipelined over the layer rotation: step i runs window_scores and select_topk of "
+                "layer i, and beside that select, without dependency waits, the decode over layer i-2's "
+                "compacted cache (TB_DECODE_CONCURRENT, max_ctas = SMs - tb_select_ctas = %d) and the "
+                "gather of layer i-1 (TB_EVICT_GATHER_CONCURRENT)" % step_ctas),
             "stage_timing": stage_timing,
             "parallelism": "replicas" if world > 1 else "single GPU"},
         "us_per_layer": {"evict": round(evict_us, 2), "decode": round(1e3 * stage_ms["decode_attn"], 2),

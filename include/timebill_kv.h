@@ -75,8 +75,8 @@ typedef enum { TB_F32 = 0, TB_BF16 = 1 } tb_dtype;
 /* Static description of a status code; never NULL. */
 const char *tb_status_string(int32_t status);
 
-/* Version of this ABI (major * 100 + minor): 102 (tb_decode_desc.max_ctas,
- * TB_DECODE_CONCURRENT, tb_select_ctas). */
+/* Version of this ABI (major * 100 + minor): 103 (tb_decode_desc.max_ctas,
+ * TB_DECODE_CONCURRENT, tb_select_ctas, TB_EVICT_GATHER_CONCURRENT). */
 int32_t tb_abi_version(void);
 
 /* Text of the last CUDA error this thread saw inside the library (the
@@ -107,6 +107,15 @@ tb_status tb_retained_count(int64_t n, int32_t window, double alpha,
  * (sum of the scores at [j - pool_k/2, j + pool_k/2] inside the prefix) /
  * pool_k, i.e. out-of-range neighbours count as zeros. */
 #define TB_EVICT_AVG_POOL 2
+/* For tb_gather_kv only (tb_score_evict ignores it: its gather waits for its
+ * own select). The caller asserts that the kernel enqueued on the stream just
+ * before the gather writes nothing the gather reads (idx, K, V), touches
+ * neither Kc nor Vc, and that idx, K and V were complete before that kernel
+ * was launched: the gather kernel then does not wait for that kernel, so,
+ * launched behind one that lets its dependents start early, it runs beside
+ * it (e.g. the gather of one layer beside the select of the next). Its
+ * completion then says nothing about that kernel's. */
+#define TB_EVICT_GATHER_CONCURRENT 4
 
 /* tb_retained_count under the TB_EVICT_BUDGET_INCLUDES_WINDOW bit of
  * `flags` (other bits are ignored here). Same errors. */

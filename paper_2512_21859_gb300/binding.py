@@ -21,7 +21,7 @@ __all__ = [
     "TbError", "EvictDesc", "DecodeDesc", "library_path", "load",
     "tb_status_string", "tb_abi_version", "tb_last_error_detail", "tb_launch_counter",
     "tb_retained_count", "tb_retained_count_ex", "TB_EVICT_BUDGET_INCLUDES_WINDOW",
-    "TB_EVICT_AVG_POOL", "TB_DECODE_EARLY_CACHE_READ", "TB_DECODE_CONCURRENT", "tb_evict_layout",
+    "TB_EVICT_AVG_POOL", "TB_EVICT_GATHER_CONCURRENT", "TB_DECODE_EARLY_CACHE_READ", "TB_DECODE_CONCURRENT", "tb_evict_layout",
     "tb_evict_workspace_size", "tb_window_scores", "tb_window_scores_lse", "tb_select_topk",
     "tb_select_ctas", "tb_gather_kv", "tb_score_evict",
     "tb_decode_workspace_size", "tb_decode_attn", "tb_read_status",
@@ -32,7 +32,7 @@ __all__ = [
 
 TB_OK, TB_ERR_INVALID_ARG, TB_ERR_UNSUPPORTED, TB_ERR_WORKSPACE, TB_ERR_CUDA, TB_ERR_TIMEOUT = range(6)
 TB_F32, TB_BF16 = 0, 1
-TB_EVICT_BUDGET_INCLUDES_WINDOW, TB_EVICT_AVG_POOL = 1, 2
+TB_EVICT_BUDGET_INCLUDES_WINDOW, TB_EVICT_AVG_POOL, TB_EVICT_GATHER_CONCURRENT = 1, 2, 4
 TB_DECODE_EARLY_CACHE_READ, TB_DECODE_CONCURRENT = 1, 2
 TB_MAX_BATCH = 64
 TB_NOALLOC_SCRATCH_BYTES = 4 << 20

@@ -26,7 +26,9 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(
   constexpr int kVecs = kRowsPerWarp * 2 * VPR;  // vectors a warp moves
   constexpr int kPerLane = kVecs / 32;
   static_assert(kPerLane <= kMaxVecPerLane, "too many vectors per lane");
-  pdl_wait();  // idx comes from the select kernel just before
+  // idx comes from the select kernel just before, unless the caller asserts
+  // (TB_EVICT_GATHER_CONCURRENT) that the kernel before writes none of it
+  if (!(p.flags & TB_EVICT_GATHER_CONCURRENT)) pdl_wait();
   pdl_trigger();
   const int b = blockIdx.y, g = blockIdx.z;
   const EvictReq& rq = p.req[b];

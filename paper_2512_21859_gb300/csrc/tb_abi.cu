@@ -69,7 +69,8 @@ bool ranges_overlap(const int64_t* off, const int64_t* len, int batch) {
 tb_status build_evict(const tb_evict_desc* d, EvictParams* p) {
   if (!d) return TB_ERR_INVALID_ARG;
   if (d->batch < 1 || d->hq < 1 || d->hkv < 1 || d->window < 1 ||
-      (d->flags & ~(TB_EVICT_BUDGET_INCLUDES_WINDOW | TB_EVICT_AVG_POOL)) != 0)
+      (d->flags & ~(TB_EVICT_BUDGET_INCLUDES_WINDOW | TB_EVICT_AVG_POOL |
+                    TB_EVICT_GATHER_CONCURRENT)) != 0)
     return TB_ERR_INVALID_ARG;
   if (d->batch > TB_MAX_BATCH) return TB_ERR_UNSUPPORTED;
   if (d->hq % d->hkv != 0) return TB_ERR_INVALID_ARG;
@@ -342,7 +343,7 @@ const char* tb_status_string(int32_t status) {
   }
 }
 
-int32_t tb_abi_version(void) { return 102; }
+int32_t tb_abi_version(void) { return 103; }
 
 const char* tb_last_error_detail(void) { return g_last_error; }
 
@@ -600,6 +601,7 @@ tb_status tb_score_evict(const tb_evict_desc* desc, const void* q_win, const voi
   float* scores = at<float>(workspace, w.scores);
   if ((st = run_window_scores(p, w, q_win, K, scores, workspace, s)) != TB_OK) return st;
   if ((st = run_select(p, w, scores, idx, pooled, workspace, s)) != TB_OK) return st;
+  p.flags &= ~TB_EVICT_GATHER_CONCURRENT;  // this gather reads the select's indices
   return cuda_status(launch_gather(p, idx, K, V, Kc, Vc, at<int32_t>(workspace, w.status), s));
 }
 

@@ -43,7 +43,7 @@ def test_status_strings_and_version(tb):
     for s in range(6):
         assert tb.tb_status_string(s)
     assert tb.tb_status_string(99) == "unknown status"
-    assert tb.tb_abi_version() == 102
+    assert tb.tb_abi_version() == 103
     assert tb.tb_last_error_detail() == ""
 
 
@@ -95,7 +95,7 @@ def test_layout_and_workspace(tb):
     (dict(kv_offset=[-1]), 1),
     (dict(out_cap=[100]), 1),                # out_cap < R
     (dict(out_rows=10), 1),
-    (dict(flags=4), 1),                      # a flag bit the library does not know
+    (dict(flags=8), 1),                      # a flag bit the library does not know
     (dict(n=[512] * 65, alpha=[0.5] * 65), 2),  # batch > TB_MAX_BATCH
     (dict(hq=2048, hkv=1), 2),               # G*W beyond the supported window rows
 ])

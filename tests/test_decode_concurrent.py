@@ -1,5 +1,6 @@
-"""The decode's CTA budget (tb_decode_desc.max_ctas) and TB_DECODE_CONCURRENT:
-a decode step that runs beside the select of another layer's eviction.
+"""The decode's CTA budget (tb_decode_desc.max_ctas), TB_DECODE_CONCURRENT and
+TB_EVICT_GATHER_CONCURRENT: a decode step, and the gather of one layer, that
+run beside the select of another layer's eviction.
 
 Checked through the C ABI:
 - with a CTA budget the keys split fewer ways; the output still matches the
@@ -11,7 +12,10 @@ Checked through the C ABI:
   stream), eagerly and replayed from a CUDA graph: the eviction's indices
   and compacted cache are bit-identical to the serial schedule's, the decode
   output is bit-identical to the same descriptor's serial call and matches
-  the oracle, and every status word stays clean.
+  the oracle, and every status word stays clean;
+- in the pipelined step (layer B's scores and select, with the decode and
+  layer A's gather beside B's select), the same bit-identity with
+  tb_score_evict per layer, which itself ignores the gather flag.
 """
 import numpy as np
 import pytest
@@ -174,3 +178,77 @@ def test_decode_beside_the_select(wl_name, n, alpha, graph):
     want = orc.decode_batch(inputs.as_f32(q, "bf16"), inputs.as_f32(Kc, "bf16"), inputs.as_f32(Vc, "bf16"),
                             lens, offs)
     assert np.max(np.abs(out.cpu().numpy() - want)) <= TOL_OUT["bf16"]
+
+
+@pytest.mark.parametrize("graph", [False, True])
+def test_gather_pipelined_beside_the_next_select(graph):
+    """TB_EVICT_GATHER_CONCURRENT in the pipelined step: layer A's scores and
+    selection, then layer B's scores and selection with, beside B's select,
+    a decode over another cache and layer A's gather (both without
+    dependency waits). Layer B is gathered last, as its own next step would.
+    Indices and compacted caches bit-identical to tb_score_evict per layer,
+    the decode output to its serial call; status words clean."""
+    wl = inputs.WORKLOADS["7b"]
+    lays = [inputs.make_layer(wl, li, alpha=0.5, n_override=[16384]) for li in (4, 5)]
+    descs = [evict_desc(wl, lay, flags=tb.TB_EVICT_GATHER_CONCURRENT) for lay in lays]
+    plain = [evict_desc(wl, lay) for lay in lays]
+    # serial reference: one tb_score_evict per layer (the flag is ignored there)
+    refs = []
+    for lay, dsc, pl in zip(lays, descs, plain):
+        r = _eviction_buffers(wl, lay, pl)
+        tb.tb_score_evict(pl, r["q_win"], r["K"], r["V"], r["idx"], r["Kc"], r["Vc"], None, r["ws"])
+        f = _eviction_buffers(wl, lay, dsc)
+        tb.tb_score_evict(dsc, f["q_win"], f["K"], f["V"], f["idx"], f["Kc"], f["Vc"], None, f["ws"])
+        torch.cuda.synchronize()
+        assert tb.tb_read_status(r["ws"]) == (tb.TB_OK, 0)
+        assert torch.equal(f["idx"], r["idx"])
+        assert torch.equal(f["Kc"].view(torch.int16), r["Kc"].view(torch.int16))
+        refs.append(r)
+    caps = [int(plain[0].out_cap[0]) + 64]
+    offs, rows, q, Kc, Vc = _cache(9, "bf16", wl.hq, wl.hkv, wl.head_dim, caps)
+    lens_d = torch.tensor([caps[0] - 3], dtype=torch.int32, device="cuda")
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=tb.TB_BF16,
+                          cache_offset=offs, cache_cap=caps, cache_rows=rows, max_len=caps[0],
+                          flags=tb.TB_DECODE_EARLY_CACHE_READ | tb.TB_DECODE_CONCURRENT,
+                          max_ctas=sms - tb.tb_select_ctas(descs[1]))
+    qd, Kd, Vd = to_dev(q, "bf16"), to_dev(Kc, "bf16"), to_dev(Vc, "bf16")
+    dws = torch.empty(tb.tb_decode_workspace_size(ddesc), dtype=torch.uint8, device="cuda")
+    tb.tb_decode_workspace_prepare(ddesc, dws)
+    ref_out = torch.empty((1, wl.hq, wl.head_dim), dtype=torch.float32, device="cuda")
+    tb.tb_decode_attn_prepared(ddesc, qd, Kd, Vd, lens_d, ref_out, dws)
+
+    bufs = [_eviction_buffers(wl, lay, dsc) for lay, dsc in zip(lays, descs)]
+    A, B = bufs
+    out = torch.full_like(ref_out, float("nan"))
+    main = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(main):
+        tb.tb_window_scores(descs[0], A["q_win"], A["K"], A["scores"], A["ws"], stream=main)
+        tb.tb_select_topk(descs[0], A["scores"], A["idx"], None, A["ws"], stream=main)
+    main.synchronize()
+
+    def step():
+        tb.tb_window_scores(descs[1], B["q_win"], B["K"], B["scores"], B["ws"], stream=main)
+        tb.tb_select_topk(descs[1], B["scores"], B["idx"], None, B["ws"], stream=main)
+        tb.tb_decode_attn_prepared(ddesc, qd, Kd, Vd, lens_d, out, dws, stream=main)
+        tb.tb_gather_kv(descs[0], A["idx"], A["K"], A["V"], A["Kc"], A["Vc"], stream=main)
+
+    if graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=main):
+            step()
+        with torch.cuda.stream(main):
+            g.replay()
+    else:
+        step()
+    main.synchronize()
+    tb.tb_gather_kv(plain[1], B["idx"], B["K"], B["V"], B["Kc"], B["Vc"])
+    torch.cuda.synchronize()
+    for buf, r in zip(bufs, refs):
+        assert tb.tb_read_status(buf["ws"]) == (tb.TB_OK, 0)
+        assert torch.equal(buf["idx"], r["idx"])
+        assert torch.equal(buf["Kc"].view(torch.int16), r["Kc"].view(torch.int16))
+        assert torch.equal(buf["Vc"].view(torch.int16), r["Vc"].view(torch.int16))
+    assert tb.tb_read_status(dws) == (tb.TB_OK, 0)
+    assert torch.equal(out, ref_out)
