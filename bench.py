@@ -522,7 +522,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
         roof["tensor"] = sroof[dom]["tensor"]
 
     lse_var = None if args.no_variants else time_lse_variant(torch, tb, dev, stream, wl, W["lay"], desc, layers,
-                                                             stage_ms, ms_step, n, peaks)
+                                                             stage_ms, ms_step, n, peaks, ab["evict"])
 
     e2e = run_e2e(args, wl, tb, torch, dev, stream, W["lay"], desc, ddesc, S["ews"], S["dws"], S["step_in"],
                   ab, R)
@@ -612,7 +612,7 @@ def window_lse_torch(torch, wl, lay, dev):
     return out
 
 
-def time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, step_ms, n, peaks):
+def time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, step_ms, n, peaks, evict_bytes):
     """tb_window_scores_lse (one QK^T pass, the window rows' normalisers
     given by the prefill) timed on the same rotated layers, and the step it
     gives with the other stages as measured."""
@@ -653,10 +653,16 @@ def time_lse_variant(torch, tb, dev, stream, wl, lay, desc, layers, stage_ms, st
     # the step with this call in place of tb_window_scores: the measured step
     # time less the difference of the two calls' stage times
     step = 1e3 * (step_ms - stage_ms["window_scores"]) + us
+    # the eviction (this call, the select and the gather, each timed alone)
+    # against the measured copy bandwidth, as the headline's eviction fraction
+    evict_us = us + 1e3 * (stage_ms["select_topk"] + stage_ms["gather_kv"])
+    evict_gbs = evict_bytes / (evict_us * 1e-6) / 1e9
     return {"call": "tb_window_scores_lse", "us": round(us, 2),
             "timing": "CUDA graph of one call per rotated layer buffer, events around the replays",
             "flops": flops, "achieved_tflops": round(tf, 1), "tensor_frac": round(tf / peak, 4),
             "step_us_with_it": round(step, 2),
+            "evict_us_with_it": round(evict_us, 2), "evict_gbs_with_it": round(evict_gbs, 1),
+            "evict_frac_with_it": round(evict_gbs / float(peaks["hbm_gbs"]), 4),
             "note": "one QK^T pass over the prefix keys; the window rows' log-sum-exp comes from the prefill"}
 
 
