@@ -320,7 +320,9 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
     # the step's decode runs beside the select (TB_DECODE_CONCURRENT) on the
     # SMs the select leaves free: its own descriptor and prepared workspaces
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    step_ctas = max(1, sms - tb.tb_select_ctas(desc))
+    step_ctas = sms - tb.tb_select_ctas(desc)
+    if step_ctas < sms // 4:  # a select that fills the GPU (many requests): the default split
+        step_ctas = 0
     sddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
                            cache_offset=desc.out_offset, cache_cap=desc.out_cap, cache_rows=desc.out_rows,
                            max_len=max(lens_h), flags=tb.TB_DECODE_EARLY_CACHE_READ | tb.TB_DECODE_CONCURRENT,
@@ -561,8 +563,9 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                 ": decode_attn, window_scores, select_topk, gather_kv" if args.serial_step else
                 ", pipelined over the layer rotation: step i runs window_scores and select_topk of "
                 "layer i, and beside that select, without dependency waits, the decode over layer i-2's "
-                "compacted cache (TB_DECODE_CONCURRENT, max_ctas = SMs - tb_select_ctas = %d) and the "
-                "gather of layer i-1 (TB_EVICT_GATHER_CONCURRENT)" % step_ctas),
+                "compacted cache (TB_DECODE_CONCURRENT, max_ctas = %s) and the gather of layer i-1 "
+                "(TB_EVICT_GATHER_CONCURRENT)" % ("SMs - tb_select_ctas = %d" % step_ctas if step_ctas
+                                                   else "0: the select fills the GPU")),
             "stage_timing": stage_timing,
             "parallelism": "replicas" if world > 1 else "single GPU"},
         "us_per_layer": {"evict": round(evict_us, 2), "decode": round(1e3 * stage_ms["decode_attn"], 2),
