@@ -12,7 +12,12 @@ namespace tb {
 namespace {
 
 constexpr int kGatherThreads = 256;
-constexpr int kRowsPerWarp = 8;
+// Four rows per warp: measured on GB300 against eight, the gather alone took
+// 128K 20.6 -> 19.6 us and 32K 13.1 -> 12.4 us, and beside a select and a
+// decode (fewer registers per block, so more blocks fit beside them) the
+// pipelined step 142.3 -> 140.5 us and 49.7 -> 47.1 us; two rows per warp, or
+// 512-thread blocks, were no better.
+constexpr int kRowsPerWarp = 4;
 constexpr int kMaxVecPerLane = 16;  // kRowsPerWarp * 2 rows * up to 32 vectors / 32 lanes
 
 // Each warp moves kRowsPerWarp retained rows of K and the matching rows of V:
