@@ -317,12 +317,16 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
     ddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
                           cache_offset=desc.out_offset, cache_cap=desc.out_cap,
                           cache_rows=desc.out_rows, max_len=max(lens_h), flags=tb.TB_DECODE_EARLY_CACHE_READ)
-    # the step's decode runs beside the select (TB_DECODE_CONCURRENT) on the
-    # SMs the select leaves free: its own descriptor and prepared workspaces
+    # the step's decode runs beside the select (TB_DECODE_CONCURRENT) on
+    # part of the SMs the select leaves free, the rest left to the gather
+    # beside it: 0.6 of them (measured on GB300, CTA budgets at 128K 88 /
+    # 72 / 56 / 40: step 140.6 / 139.8 / 140.0 / 141.3 us; at 32K 120 / 96 /
+    # 72 / 48: 47.3 / 46.7 / 45.8 / 48.6 us); its own descriptor and
+    # prepared workspaces
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    step_ctas = sms - tb.tb_select_ctas(desc)
-    if step_ctas < sms // 4:  # a select that fills the GPU (many requests): the default split
-        step_ctas = 0
+    free = sms - tb.tb_select_ctas(desc)
+    # a select that fills the GPU (many requests): the default split
+    step_ctas = int(0.6 * free + 0.5) if free >= sms // 4 else 0
     sddesc = tb.DecodeDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, dtype=desc.dtype,
                            cache_offset=desc.out_offset, cache_cap=desc.out_cap, cache_rows=desc.out_rows,
                            max_len=max(lens_h), flags=tb.TB_DECODE_EARLY_CACHE_READ | tb.TB_DECODE_CONCURRENT,
@@ -564,7 +568,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                 ", pipelined over the layer rotation: step i runs window_scores and select_topk of "
                 "layer i, and beside that select, without dependency waits, the decode over layer i-2's "
                 "compacted cache (TB_DECODE_CONCURRENT, max_ctas = %s) and the gather of layer i-1 "
-                "(TB_EVICT_GATHER_CONCURRENT)" % ("SMs - tb_select_ctas = %d" % step_ctas if step_ctas
+                "(TB_EVICT_GATHER_CONCURRENT)" % ("0.6 x (SMs - tb_select_ctas) = %d" % step_ctas if step_ctas
                                                    else "0: the select fills the GPU")),
             "stage_timing": stage_timing,
             "parallelism": "replicas" if world > 1 else "single GPU"},
