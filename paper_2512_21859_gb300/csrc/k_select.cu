@@ -433,17 +433,14 @@ __global__ void __launch_bounds__(kCsThreads) select_cluster_kernel(
   // no shared memory of another CTA is read after this point: arrive now, and
   // wait (so that none leaves while another may still read it) at the end
   asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
-  // offsets of this CTA: ties are kept in index order until `need` are in
-  int eqbase = 0, selbase = 0;
-  for (int r = 0; r < rank; ++r) {
-    const int tg = sh.rank_cnt[r][0], te = sh.rank_cnt[r][1];
-    selbase += tg + max(0, min(need - eqbase, te));
-    eqbase += te;
-  }
-  for (int w = 0; w < warp; ++w) {
-    selbase += sh.wgt[w] + max(0, min(need - eqbase, sh.weq[w]));
-    eqbase += sh.weq[w];
-  }
+  // offsets of this warp: ties are kept in index order until `need` are in,
+  // so of the E ties before a point min(need, E) are kept, and the offsets
+  // are prefix sums of the lower ranks' and warps' counts (one reduction
+  // each, no chain through the warps)
+  const int lg = (lane < rank ? sh.rank_cnt[lane & 7][0] : 0) + (lane < warp ? sh.wgt[lane] : 0);
+  const int le = (lane < rank ? sh.rank_cnt[lane & 7][1] : 0) + (lane < warp ? sh.weq[lane] : 0);
+  int eqbase = __reduce_add_sync(0xffffffffu, le);
+  int selbase = __reduce_add_sync(0xffffffffu, lg) + min(need, eqbase);
   if (k > 0) {
     // emission from the count pass's ballots: per 32-key chunk, the keys
     // above tau and the first ties until `need` of them are kept
