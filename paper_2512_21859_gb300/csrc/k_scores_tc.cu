@@ -17,11 +17,11 @@
 //                       reading the key tiles in reverse order so that the
 //                       tail pass 1 loaded last is still in L2. The four
 //                       quarter sums of a key meet in global memory: the launch
-//                       that runs pass 1 clears the scores first, and each warp
-//                       adds its sum with a reduction (no hand-off between the
-//                       warps of a lane quadrant). The votes-only launch fed by
-//                       the prefill's log-sum-exp sums the quarters through
-//                       shared memory instead, in a fixed order.
+//                       that runs pass 1 clears the scores first (for the
+//                       votes-only launch fed by the prefill's log-sum-exp, the
+//                       caller's clearing kernel does), and each warp adds its
+//                       sum with a reduction (no hand-off between the warps of
+//                       a lane quadrant).
 //
 // One kernel template runs pass 1, pass 2, or both. Both (the default) is a
 // cooperative launch of one CTA per SM: after pass 1 every CTA publishes its
@@ -74,10 +74,12 @@ constexpr int kSumMinChunks = 24;
 // kRedVotes: the launch that runs pass 1 zeroes the scores as it starts, and
 // pass 2's warps add their quarter sums of the window rows into them with
 // global reductions (no hand-off between the four warps of a lane quadrant).
-// Measured on GB300 (128K, per call): 114.8 -> 108.7 us, with each warp's
-// reduction issued after its next TMEM load wait and relaxed hand-back
-// arrivals (issued before the wait, or behind a release arrival, the stores
-// stalled the warp: 134 us).
+// Every launch that runs pass 2 carries it (the votes-only launch adds into
+// scores its caller cleared). Measured on GB300 (128K, per call): against a
+// shared-memory hand-off, 114.8 -> 108.7 us for both passes and 64.8 ->
+// 59.1 us for the votes-only launch, with each warp's reduction issued after
+// its next TMEM load wait and relaxed hand-back arrivals (issued before the
+// wait, or behind a release arrival, the stores stalled the warp: 134 us).
 enum : int { kPassStats = 1, kPassVotes = 2, kPassBoth = 3, kRowSums = 4, kRedVotes = 8 };
 
 template <int D>
@@ -90,8 +92,7 @@ struct Geo {
   static constexpr int kRingOff = kQBytes;
   static constexpr int kBarOff = kRingOff + kStages * kTileBytes;
   static constexpr int kCrOff = kBarOff + 1024;          // -c_row for 256 rows
-  static constexpr int kXOff = kCrOff + 256 * 4;         // pass 2: 2 x 3 x 128 partial sums
-  static constexpr int kMOff = kXOff + 2 * 3 * 128 * 4;  // pass 1: 256 (max, sum) pairs
+  static constexpr int kMOff = kCrOff + 256 * 4;         // pass 1: 256 (max, sum) pairs
   static constexpr int kSmem = kMOff + 256 * 8 + 1024;   // + alignment slack
 };
 
@@ -101,8 +102,6 @@ struct Bars {
   uint64_t tfull[2];
   uint64_t tempty[2];
   uint64_t qfull;
-  uint64_t xfull[2][4];  // pass 2, per lane quadrant: the other quarters' sums are in xbuf
-  uint64_t xempty[2][4];
   uint64_t mrg;       // pass 1: the second column halves wrote their (max, sum)
   uint64_t pub;       // both passes: the CTA's partials are written
   uint64_t gready;    // both passes: every CTA of the grid published
@@ -241,7 +240,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* ring = smem + G::kRingOff;
   Bars* bars = reinterpret_cast<Bars*>(smem + G::kBarOff);
   float* ncr = reinterpret_cast<float*>(smem + G::kCrOff);
-  float* xbuf = reinterpret_cast<float*>(smem + G::kXOff);
   float2* mrg = reinterpret_cast<float2*>(smem + G::kMOff);
 
   const int item = blockIdx.x;
@@ -261,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const size_t segrow = ((size_t)info.b * p.hkv + info.g) * M;
   constexpr bool kFused = (MODE & kPassBoth) == kPassBoth;
   constexpr bool kSums = kFused && (MODE & kRowSums) != 0;
-  constexpr bool kRed = (MODE & kRedVotes) != 0;
+  static_assert(!(MODE & kPassVotes) || (MODE & kRedVotes), "pass 2 adds by reductions");
   float* const sc_out = scores + (size_t)info.g * p.score_rows + rq.score_off;
 
 
@@ -274,10 +272,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(&bars->tfull[a], 1);
       tc::mbar_init(&bars->tempty[a], kEpiWarps);
-      for (int qd = 0; qd < 4; ++qd) {
-        tc::mbar_init(&bars->xfull[a][qd], 3);
-        tc::mbar_init(&bars->xempty[a][qd], 1);
-      }
     }
     tc::mbar_init(&bars->qfull, 1);
     tc::mbar_init(&bars->mrg, kEpiWarps / 2);
@@ -294,7 +288,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // global memory from here on (the votes-only launch is a programmatic
   // dependent launch: its set-up above overlapped the previous kernel)
   pdl_wait();
-  if (kRed && (MODE & kPassStats)) {
+  if ((MODE & kRedVotes) && (MODE & kPassStats)) {
     // the launch that runs pass 1 clears every score before any pass 2 tile
     // adds into it (the grid barrier, or the launch boundary, orders the two);
     // these stores go out while the first key tiles are on their way
@@ -604,9 +598,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if ((MODE & kPassVotes) && ok) {
       // keys: TMEM lane quadrant quad; window rows (columns): quarter `sub`
       const int key = quad * 32 + lane;  // TMEM lane = key within the tile
-      int pend_j = -1;  // a score store (or reduction) not yet issued
+      int pend_j = -1;  // a reduction not yet issued
       float pend_v = 0.f;
-      for (int it2 = 0;; ++it2, ++it) {
+      for (;; ++it) {
         const int a = it & 1;
         if (!tc::mbar_wait(&bars->tfull[a], (it >> 1) & 1, abort, status)) break;
         tc::tc_fence_after();
@@ -624,11 +618,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::tmem_ld32(taddr + c0, *reinterpret_cast<float(*)[32]>(v));
           if (c0 + 32 < NP) tc::tmem_ld32(taddr + c0 + 32, *reinterpret_cast<float(*)[32]>(v + 32));
           tc::tmem_ld_wait();
-          // the previous tile's score store or reduction, issued after this
-          // wait (a TMEM load wait issued behind a global store waits for it)
+          // the previous tile's reduction, issued after this wait (a TMEM
+          // load wait issued behind a global store waits for it)
           if (pend_j >= 0) {
-            if (kRed) atomicAdd(sc_out + pend_j, pend_v);
-            else sc_out[pend_j] = pend_v;
+            atomicAdd(sc_out + pend_j, pend_v);
             pend_j = -1;
           }
           tc::tc_fence_before();
@@ -648,41 +641,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) tc::mbar_arrive_rx(&bars->tempty[a]);
         }
-        if (kRed) {
-          // this warp's quarter of the window rows, added into the key's score
-          const int j = t * kTileKeys + key;
-          if (sub * 64 < NP && j < rq.p) {
-            pend_j = j;
-            pend_v = acc;
-          }
-          continue;
-        }
-        // combine the four quarters of the window rows through a double-buffered
-        // hand-off between the four warps of this lane quadrant (one SM
-        // sub-partition; bounded mbarrier waits, no named barrier); fixed sum order
-        const int x = it2 & 1;
-        const uint32_t xph = (uint32_t)((it2 >> 1) & 1);
-        if (sub > 0) {
-          if (!tc::mbar_wait(&bars->xempty[x][quad], xph ^ 1, abort, status)) break;
-          xbuf[(x * 3 + sub - 1) * 128 + key] = acc;
-          __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&bars->xfull[x][quad]);
-        } else {
-          if (!tc::mbar_wait(&bars->xfull[x][quad], xph, abort, status)) break;
-          const int j = t * kTileKeys + key;
-          const float* xb = xbuf + x * 3 * 128;
-          if (j < rq.p) {
-            pend_j = j;
-            pend_v = ((acc + xb[key]) + xb[128 + key]) + xb[256 + key];
-          }
-          __syncwarp();
-          if (lane == 0) tc::mbar_arrive_rx(&bars->xempty[x][quad]);
+        // this warp's quarter of the window rows, added into the key's score
+        const int j = t * kTileKeys + key;
+        if (sub * 64 < NP && j < rq.p) {
+          pend_j = j;
+          pend_v = acc;
         }
       }
-      if (pend_j >= 0) {
-        if (kRed) atomicAdd(sc_out + pend_j, pend_v);
-        else sc_out[pend_j] = pend_v;
-      }
+      if (pend_j >= 0) atomicAdd(sc_out + pend_j, pend_v);
     }
   }
 
@@ -866,8 +832,9 @@ cudaError_t launch_window_votes_tc(const EvictParams& p, const void* q_win, cons
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   };
-  return p.d == 64 ? launch(ws_tc<64, kPassVotes>, Geo<64>::kSmem)
-                   : launch(ws_tc<128, kPassVotes>, Geo<128>::kSmem);
+  // the caller cleared the scores (with the workspace's control words)
+  return p.d == 64 ? launch(ws_tc<64, kPassVotes | kRedVotes>, Geo<64>::kSmem)
+                   : launch(ws_tc<128, kPassVotes | kRedVotes>, Geo<128>::kSmem);
 }
 
 bool window_scores_row_sums(const EvictParams& p) {

@@ -296,6 +296,34 @@ __global__ void clear_words(uint4* __restrict__ w, size_t n16) {
     w[i] = make_uint4(0u, 0u, 0u, 0u);
 }
 
+// The same, and the nf floats at f (16-byte aligned) as well: the scores the
+// votes-only scoring adds into, in the same launch.
+__global__ void clear_words_and_floats(uint4* __restrict__ w, size_t n16, float* __restrict__ f,
+                                       size_t nf) {
+  pdl_wait();
+  pdl_trigger();
+  const size_t nf16 = nf / 4, total = n16 + nf16;
+  uint4* f4 = reinterpret_cast<uint4*>(f);
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    if (i < n16) w[i] = make_uint4(0u, 0u, 0u, 0u);
+    else f4[i - n16] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < (nf & 3)) f[nf16 * 4 + threadIdx.x] = 0.f;
+}
+
+cudaError_t clear_control_words_and_floats(void* ws, size_t bytes, float* f, size_t nf,
+                                           cudaStream_t s) {
+  const size_t n16 = bytes / 16;  // callers pass multiples of 256 bytes
+  const size_t total = n16 + nf / 4 + 1;
+  const unsigned blocks = (unsigned)std::min<size_t>((total + 255) / 256, 152);
+  const cudaError_t e = launch_pdl(clear_words_and_floats, dim3(blocks), dim3(256), 0, s,
+                                   static_cast<uint4*>(ws), n16, f, nf);
+  count_launches(1);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t clear_control_words(void* ws, size_t bytes, cudaStream_t s) {
@@ -537,7 +565,14 @@ tb_status tb_window_scores_lse(const tb_evict_desc* desc, const void* q_win, con
   const EvictWorkspace w = carve_evict(p);
   if ((st = check_ws(workspace, workspace_bytes, w.total)) != TB_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = cuda_status(clear_control_words(workspace, evict_clear_bytes(p, w), s))) != TB_OK) return st;
+  // the tensor-core votes kernel adds the quarters of each key's sum into the
+  // scores, so it gets them cleared with the control words
+  if (window_scores_tc_supported(p))
+    st = cuda_status(clear_control_words_and_floats(workspace, evict_clear_bytes(p, w), scores,
+                                                    (size_t)p.hkv * (size_t)p.score_rows, s));
+  else
+    st = cuda_status(clear_control_words(workspace, evict_clear_bytes(p, w), s));
+  if (st != TB_OK) return st;
   p.rowc_scale = 1.4426950408889634f;  // natural-log LSE -> log2 units
   return cuda_status(launch_window_votes(p, q_win, K, scores, lse, at<int32_t>(workspace, w.status),
                                          at<int32_t>(workspace, w.tilectr), s));
