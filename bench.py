@@ -3,14 +3,16 @@
 
 One step = one transformer layer of the path: one decode step of attention
 over a compacted cache (tb_decode_attn_prepared: the decode workspace is
-prepared once, as a decode loop keeps it) and the layer's prompt-time
+prepared once, as a decode loop keeps it) and a layer's prompt-time
 eviction (tb_window_scores -> tb_select_topk -> tb_gather_kv, the stages
-tb_score_evict chains), enqueued as scoring, select, decode, gather: the
-decode's CTAs start during the select on the SMs it leaves free, and attend
-over the cache the previous step's eviction wrote (--serial-step: decode
-first, over the buffer's own cache from one rotation earlier). Layers rotate
-over enough device buffers that every step's inputs are larger than L2
-(129 MB), so no step reads another step's data from cache.
+tb_score_evict chains), pipelined over the layer rotation: step i scores
+layer i and selects its rows, and beside that select run the decode over
+layer i-2's compacted cache and the gather of layer i-1, both without
+dependency waits (TB_DECODE_CONCURRENT with a CTA budget,
+TB_EVICT_GATHER_CONCURRENT). --serial-step: decode first, then the eviction,
+on one stream. Layers rotate over enough device buffers that every step's
+inputs are larger than L2 (129 MB), so no step reads another step's data
+from cache.
 
 Prints ONE JSON line. value = algorithmic HBM bytes of the step (K read once
 to score, retained K/V rows read and written, compacted K/V read by decode)
