@@ -848,7 +848,12 @@ def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_i
         ms = timed(overlapped)
         st, raw = tb.tb_read_status(hws, stream=stream)
         assert st == tb.TB_OK, raw
-        same_idx = bool(torch.equal(idx_h, idx_serial))
+        # the share of retained positions the per-head and the batched calls
+        # agree on (the scores' float-atomic sums vary in their last bit from
+        # run to run, so keys tied with the k-th threshold can swap)
+        a, b = idx_h.numpy(), idx_serial.numpy()
+        same_idx = round(float(np.mean([np.intersect1d(a[g], b[g]).size / max(1, a.shape[1])
+                                        for g in range(a.shape[0])])), 6)
     ms_copy = timed(copy_only)
     h2d = sum(v.numel() * v.element_size() for v in h.values()) + sum(
         v.numel() * v.element_size() for v in (hq, hk, hv))
@@ -861,7 +866,7 @@ def run_e2e(args, wl, tb, torch, dev, stream, lay, desc, ddesc, ews, dws, step_i
             "copy_only_ms_per_step": round(ms_copy, 4),
             "pinned_h2d_gbs": round(h2d / (ms_copy * 1e-3) / 1e9, 1),
             "copy_bound_frac": round(ms_copy / ms, 4),
-            "per_head_idx_equal_batched": same_idx}
+            "per_head_idx_agreement_with_batched": same_idx}
 
 
 def describe(wl, n, a):
