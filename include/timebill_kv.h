@@ -113,8 +113,10 @@ tb_status tb_retained_count(int64_t n, int32_t window, double alpha,
  * neither Kc nor Vc, and that idx, K and V were complete before that kernel
  * was launched: the gather kernel then does not wait for that kernel, so,
  * launched behind one that lets its dependents start early, it runs beside
- * it (e.g. the gather of one layer beside the select of the next). Its
- * completion then says nothing about that kernel's. */
+ * it (e.g. the gather of one layer beside the select of the next). One of
+ * its threads still waits for that kernel before it exits, so the gather
+ * completes only after that kernel has: work ordered after the gather is
+ * ordered after both. */
 #define TB_EVICT_GATHER_CONCURRENT 4
 
 /* tb_retained_count under the TB_EVICT_BUDGET_INCLUDES_WINDOW bit of
@@ -248,9 +250,9 @@ tb_status tb_score_evict(const tb_evict_desc *desc, const void *q_win,
  * lets its dependents start early (the library's select and gather kernels
  * do, right after their own dependency wait), it runs beside it on the SMs
  * that kernel leaves free (size it with max_ctas, e.g. the SM count minus
- * tb_select_ctas). The call's completion then says nothing about that
- * work's: whatever needs the preceding kernel's results must be ordered
- * after it by an event recorded before this call. Implies
+ * tb_select_ctas). One of its threads still waits for the preceding
+ * kernel before it exits, so the call completes only after that kernel
+ * has: work ordered after the call is ordered after both. Implies
  * TB_DECODE_EARLY_CACHE_READ. No effect on tb_decode_attn and
  * tb_decode_attn_noalloc (their clearing kernel comes first). */
 #define TB_DECODE_CONCURRENT 2

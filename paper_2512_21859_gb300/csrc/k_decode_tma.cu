@@ -236,13 +236,12 @@ __device__ __forceinline__ void merge_splits(const DecodeParams& p, int b, int g
 }
 
 template <int D, int G>
-__global__ void __launch_bounds__(kThreads, 1)
-    decode_tma(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tk,
-               const __grid_constant__ CUtensorMap tv, const uint16_t* __restrict__ kc,
-               const uint16_t* __restrict__ vc, const uint16_t* __restrict__ q,
-               const int32_t* __restrict__ lens, float* __restrict__ part_o,
-               float2* __restrict__ part_ml, int32_t* __restrict__ counters,
-               void* __restrict__ out, int32_t* __restrict__ status) {
+__device__ __forceinline__ void decode_tma_body(
+    const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
+    const uint16_t* __restrict__ kc, const uint16_t* __restrict__ vc,
+    const uint16_t* __restrict__ q, const int32_t* __restrict__ lens, float* __restrict__ part_o,
+    float2* __restrict__ part_ml, int32_t* __restrict__ counters, void* __restrict__ out,
+    int32_t* __restrict__ status) {
   using Gm = DGeo<D>;
   constexpr int KS = D / 16;  // k-steps of Q K^T
   constexpr int NT = D / 8;   // n-tiles of P V
@@ -293,7 +292,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   // by the preceding kernel) is read again after the wait, below. Mode 3:
   // the caller asserts that the preceding kernel writes nothing this one
   // reads and that everything it reads was complete before that kernel was
-  // launched, so there is no wait at all and this kernel runs beside it.
+  // launched, so there is no wait before the work and this kernel runs
+  // beside it (one thread waits for it at the very end, below).
   // Without either (a prepared workspace, no assertion) any kernel may
   // precede this one, so the requests wait for it.
   int issued = 0;
@@ -587,6 +587,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (!*last_flag) return;
   merge_splits<D, G, 1>(p, b, g, 0, part_o, part_ml, out, status, reinterpret_cast<float*>(smem), len);
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(kThreads, 1)
+    decode_tma(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tk,
+               const __grid_constant__ CUtensorMap tv, const uint16_t* __restrict__ kc,
+               const uint16_t* __restrict__ vc, const uint16_t* __restrict__ q,
+               const int32_t* __restrict__ lens, float* __restrict__ part_o,
+               float2* __restrict__ part_ml, int32_t* __restrict__ counters,
+               void* __restrict__ out, int32_t* __restrict__ status) {
+  decode_tma_body<D, G>(p, tk, tv, kc, vc, q, lens, part_o, part_ml, counters, out, status);
+  // Mode 3 never waited for the preceding kernel: one thread waits for it
+  // now, after all of this CTA's work, so that this grid completes only after
+  // that kernel has. Whatever waits for this grid (the merge kernel, the next
+  // kernel's own dependency wait, the stream) then waits for both. The
+  // preceding kernel's CTAs are all resident by now (it let this grid launch
+  // only once every one of them had started), so the wait ends.
+  if (p.early_tma == 3 && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0)
+    pdl_wait();
 }
 
 // The split merge as a kernel of its own, kMergeParts CTAs per (KV head,

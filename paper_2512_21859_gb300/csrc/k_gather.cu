@@ -24,17 +24,13 @@ constexpr int kMaxVecPerLane = 16;  // kRowsPerWarp * 2 rows * up to 32 vectors 
 // first every lane issues all of its 16-byte loads, then all of its stores,
 // so that each lane keeps several independent loads in flight.
 template <int VPR>
-__global__ void __launch_bounds__(kGatherThreads) gather_kernel(
-    const __grid_constant__ EvictParams p, const int32_t* __restrict__ idx,
-    const uint4* __restrict__ K, const uint4* __restrict__ V, uint4* __restrict__ Kc,
-    uint4* __restrict__ Vc, int32_t* __restrict__ status) {
+__device__ __forceinline__ void gather_rows(const EvictParams& p, const int32_t* __restrict__ idx,
+                                            const uint4* __restrict__ K, const uint4* __restrict__ V,
+                                            uint4* __restrict__ Kc, uint4* __restrict__ Vc,
+                                            int32_t* __restrict__ status) {
   constexpr int kVecs = kRowsPerWarp * 2 * VPR;  // vectors a warp moves
   constexpr int kPerLane = kVecs / 32;
   static_assert(kPerLane <= kMaxVecPerLane, "too many vectors per lane");
-  // idx comes from the select kernel just before, unless the caller asserts
-  // (TB_EVICT_GATHER_CONCURRENT) that the kernel before writes none of it
-  if (!(p.flags & TB_EVICT_GATHER_CONCURRENT)) pdl_wait();
-  pdl_trigger();
   const int b = blockIdx.y, g = blockIdx.z;
   const EvictReq& rq = p.req[b];
   const int R = rq.k + p.window;
@@ -68,6 +64,26 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(
     uint4* dst = (w < VPR ? Kc : Vc) + dst_base + (size_t)(r0 + rr) * VPR + (w < VPR ? w : w - VPR);
     *dst = buf[i];
   }
+}
+
+template <int VPR>
+__global__ void __launch_bounds__(kGatherThreads) gather_kernel(
+    const __grid_constant__ EvictParams p, const int32_t* __restrict__ idx,
+    const uint4* __restrict__ K, const uint4* __restrict__ V, uint4* __restrict__ Kc,
+    uint4* __restrict__ Vc, int32_t* __restrict__ status) {
+  // idx comes from the select kernel just before, unless the caller asserts
+  // (TB_EVICT_GATHER_CONCURRENT) that the kernel before writes none of it
+  const bool concurrent = p.flags & TB_EVICT_GATHER_CONCURRENT;
+  if (!concurrent) pdl_wait();
+  pdl_trigger();
+  gather_rows<VPR>(p, idx, K, V, Kc, Vc, status);
+  // A concurrent gather waits for the kernel before it only now, in one
+  // thread after all of its block's copies, so that the grid still completes
+  // after that kernel: whatever waits for the gather waits for both. That
+  // kernel's CTAs have all started (it let this grid launch only then), so
+  // the wait ends.
+  if (concurrent && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0)
+    pdl_wait();
 }
 
 }  // namespace

@@ -63,8 +63,9 @@ struct DecodeParams {
   // dependency wait; 2: the same on the caller's word (prepared workspace
   // with TB_DECODE_EARLY_CACHE_READ) that the work before it writes no cache
   // row below lens[b] - 1, which is read again after the wait; 3
-  // (TB_DECODE_CONCURRENT): no dependency wait at all, the work before it
-  // writes nothing the decode reads; 0 (prepared workspaces otherwise):
+  // (TB_DECODE_CONCURRENT): no dependency wait before the work (the work
+  // before it writes nothing the decode reads), one thread waits at the end
+  // so that the grid still completes after it; 0 (prepared workspaces otherwise):
   // anything may precede it
   int32_t early_tma;
   int64_t cache_rows;

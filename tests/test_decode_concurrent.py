@@ -9,7 +9,9 @@ Checked through the C ABI:
 - in the schedule the flag is for (window scores, select, then the decode as
   the select's programmatic dependent, sized to the SMs the select leaves
   free, with the gather ordered after the select by an event on a second
-  stream), eagerly and replayed from a CUDA graph: the decode output is
+  stream, or simply after the decode on the same stream, since the decode
+  grid completes only after the select), eagerly and replayed from a CUDA
+  graph: the decode output is
   bit-identical to the same descriptor's serial call and matches the oracle,
   and every status word stays clean;
 - in the pipelined step (layer B's scores and select, with the decode and
@@ -146,7 +148,11 @@ def _gathered(buf, desc):
 
 @pytest.mark.parametrize("wl_name,n,alpha", [("7b", 16384, 0.5), ("128k", 40000, 0.9)])
 @pytest.mark.parametrize("graph", [False, True])
-def test_decode_beside_the_select(wl_name, n, alpha, graph):
+@pytest.mark.parametrize("order", ["side_stream", "same_stream"])
+def test_decode_beside_the_select(wl_name, n, alpha, graph, order):
+    """order "same_stream": the gather of the select's rows comes right after
+    the concurrent decode on the one stream, ordered after the select only by
+    the decode grid completing after it (its deferred dependency wait)."""
     wl = inputs.WORKLOADS[wl_name]
     lay = inputs.make_layer(wl, 3, alpha=alpha, n_override=[n])
     desc = evict_desc(wl, lay)
@@ -185,10 +191,14 @@ def test_decode_beside_the_select(wl_name, n, alpha, graph):
     def schedule():
         tb.tb_window_scores(desc, con["q_win"], con["K"], con["scores"], con["ws"], stream=main)
         tb.tb_select_topk(desc, con["scores"], con["idx"], None, con["ws"], stream=main)
-        side.wait_stream(main)        # the gather after the select's completion
+        if order == "side_stream":
+            side.wait_stream(main)    # the gather after the select's completion
         tb.tb_decode_attn_prepared(ddesc, qd, Kd, Vd, lens_d, out, dws, stream=main)
-        tb.tb_gather_kv(desc, con["idx"], con["K"], con["V"], con["Kc"], con["Vc"], stream=side)
-        main.wait_stream(side)
+        if order == "side_stream":
+            tb.tb_gather_kv(desc, con["idx"], con["K"], con["V"], con["Kc"], con["Vc"], stream=side)
+            main.wait_stream(side)
+        else:
+            tb.tb_gather_kv(desc, con["idx"], con["K"], con["V"], con["Kc"], con["Vc"], stream=main)
 
     torch.cuda.synchronize()
     if graph:
