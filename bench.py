@@ -49,7 +49,7 @@ NOMINAL_HBM_GBS = 8000.0
 # the metric's alpha axis, carried in the one JSON line of every run
 ALPHA_SWEEP = [("128k", (0.5, 0.75, 0.9)), ("32k", (0.0, 0.25, 0.5, 0.75, 0.9, 0.95))]
 # the algorithmic bytes of each stage per launch (the method's minimum)
-SURVEY_BYTES_RULE = {
+ALG_BYTES_RULE = {
     "window_scores": "e Hkv d sum(N) + q_win bytes: K read once",
     "select_topk": "4 Hkv (2 sum(P) + sum(R)): scores read, pooled written, indices written",
     "gather_kv": "4 e Hkv d sum(R): retained K and V rows read and written",
@@ -545,7 +545,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
             "traffic": profiled_traffic(dom, wl.name),
             "alg_bytes_per_launch": int(ab[dom]), "avg_launch_ms": round(stage_ms[dom], 5),
-            "bytes_rule": SURVEY_BYTES_RULE.get(dom, "")}
+            "bytes_rule": ALG_BYTES_RULE.get(dom, "")}
     if "tensor" in sroof.get(dom, {}):
         roof["tensor"] = sroof[dom]["tensor"]
 
