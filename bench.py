@@ -323,8 +323,10 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
     # part of the SMs the select leaves free, the rest left to the gather
     # beside it: 0.6 of them (measured on GB300, CTA budgets at 128K 88 /
     # 72 / 56 / 40: step 140.6 / 139.8 / 140.0 / 141.3 us; at 32K 120 / 96 /
-    # 72 / 48: 47.3 / 46.7 / 45.8 / 48.6 us); its own descriptor and
-    # prepared workspaces
+    # 72 / 48: 47.3 / 46.7 / 45.8 / 48.6 us; as fractions of the free SMs,
+    # 0.4 / 0.5 / 0.6 / 0.7 / 0.8 at 128K: 144.2 / 139.6 / 136.6 / 136.6 /
+    # 136.5 us, at 32K: 44.7 / 42.8 / 42.4 / 42.4 / 42.4 us); its own
+    # descriptor and prepared workspaces
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     free = sms - tb.tb_select_ctas(desc)
     # a select that fills the GPU (many requests): the default split
