@@ -149,16 +149,20 @@ def _gathered(buf, desc):
 @pytest.mark.parametrize("wl_name,n,alpha", [("7b", 16384, 0.5), ("128k", 40000, 0.9)])
 @pytest.mark.parametrize("graph", [False, True])
 @pytest.mark.parametrize("order", ["side_stream", "same_stream"])
-def test_decode_beside_the_select(wl_name, n, alpha, graph, order):
+@pytest.mark.parametrize("cache", ["long", "short"])
+def test_decode_beside_the_select(wl_name, n, alpha, graph, order, cache):
     """order "same_stream": the gather of the select's rows comes right after
     the concurrent decode on the one stream, ordered after the select only by
-    the decode grid completing after it (its deferred dependency wait)."""
+    the decode grid completing after it (its deferred dependency wait).
+    cache "short": 2048 rows, so that every split is one 128-key tile and a
+    merge kernel follows the split kernel (the deferred wait is then in the
+    first of the two)."""
     wl = inputs.WORKLOADS[wl_name]
     lay = inputs.make_layer(wl, 3, alpha=alpha, n_override=[n])
     desc = evict_desc(wl, lay)
     # the decode attends over another layer's compacted cache, as in a step
     # that evicts one layer while it decodes the previous one
-    caps = [int(desc.out_cap[0]) + 64]
+    caps = [int(desc.out_cap[0]) + 64] if cache == "long" else [2048]
     offs, rows, q, Kc, Vc = _cache(7, "bf16", wl.hq, wl.hkv, wl.head_dim, caps)
     lens = [caps[0] - 5]
     sms = torch.cuda.get_device_properties(0).multi_processor_count
