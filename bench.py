@@ -309,7 +309,7 @@ def setup_alpha(torch, tb, W, alpha_vec, rank, dev, stream):
                         pool_k=wl.pool_k, dtype=tb.TB_BF16 if wl.dtype == "bf16" else tb.TB_F32,
                         n=n, alpha=alpha_vec, kv_offset=lay["kv_offset"], kv_rows=int(np.sum(n)),
                         out_cap=lens_h)
-    # the step's gather runs beside the next layer's select (no dependency wait)
+    # the step's gather runs beside the next layer's select (no dependency wait before its copies)
     gdesc = tb.EvictDesc(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, window=wl.window,
                          pool_k=wl.pool_k, dtype=desc.dtype, n=n, alpha=alpha_vec, kv_offset=lay["kv_offset"],
                          kv_rows=int(np.sum(n)), out_cap=lens_h, flags=tb.TB_EVICT_GATHER_CONCURRENT)
@@ -455,7 +455,7 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
     # each layer buffer's step captured into a CUDA graph of the four calls,
     # pipelined over the layer rotation: step i scores layer i and selects
     # its rows; beside that select (bound by the latency of its phases on
-    # the SMs its clusters hold) run, without dependency waits, the decode
+    # the SMs its clusters hold) run, without waiting for it first, the decode
     # over layer i-2's compacted cache (TB_DECODE_CONCURRENT, a CTA budget
     # of the SMs the select leaves free) and the gather of layer i-1 (its
     # rows selected in step i-1; TB_EVICT_GATHER_CONCURRENT), both bound by
@@ -585,13 +585,13 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
                     "pipelined, the gather and the decode are of the previous layers (see launch)",
             "decode_call": "tb_decode_attn_prepared with TB_DECODE_EARLY_CACHE_READ (workspace prepared once; "
                            "no per-call clearing kernel; first tiles requested before the preceding kernel ends); "
-                           "in the step also with TB_DECODE_CONCURRENT and max_ctas (no dependency wait: it "
-                           "runs beside the select)",
+                           "in the step also with TB_DECODE_CONCURRENT and max_ctas (no dependency wait before its "
+                           "work: it runs beside the select)",
             "launch": "the steps replay a CUDA graph of a whole rotation of %d steps (one-step graphs for "
                       "any remainder of the K steps), each step the four C-ABI calls" % L + (
                 ": decode_attn, window_scores, select_topk, gather_kv" if args.serial_step else
                 ", pipelined over the layer rotation: step i runs window_scores and select_topk of "
-                "layer i, and beside that select, without dependency waits, the decode over layer i-2's "
+                "layer i, and beside that select, without waiting for it first, the decode over layer i-2's "
                 "compacted cache (TB_DECODE_CONCURRENT, max_ctas = %s) and the gather of layer i-1 "
                 "(TB_EVICT_GATHER_CONCURRENT)" % ("0.6 x (SMs - tb_select_ctas) = %d" % step_ctas if step_ctas
                                                    else "0: the select fills the GPU")),

@@ -111,9 +111,10 @@ tb_status tb_retained_count(int64_t n, int32_t window, double alpha,
  * own select). The caller asserts that the kernel enqueued on the stream just
  * before the gather writes nothing the gather reads (idx, K, V), touches
  * neither Kc nor Vc, and that idx, K and V were complete before that kernel
- * was launched: the gather kernel then does not wait for that kernel, so,
- * launched behind one that lets its dependents start early, it runs beside
- * it (e.g. the gather of one layer beside the select of the next). One of
+ * was launched: the gather kernel then does not wait for that kernel before
+ * its copies, so, launched behind one that lets its dependents start early,
+ * it runs beside it (e.g. the gather of one layer beside the select of the
+ * next). One of
  * its threads still waits for that kernel before it exits, so the gather
  * completes only after that kernel has: work ordered after the gather is
  * ordered after both. */
@@ -246,7 +247,7 @@ tb_status tb_score_evict(const tb_evict_desc *desc, const void *q_win,
  * tb_decode_attn_prepared call writes nothing the call reads (q, Kc, Vc,
  * lens) and touches neither out nor the workspace, and that everything the
  * call reads was complete before that work was launched. The decode kernel
- * then does not wait for that work at all: launched behind a kernel that
+ * then does not wait for that work before its own: launched behind a kernel that
  * lets its dependents start early (the library's select and gather kernels
  * do, right after their own dependency wait), it runs beside it on the SMs
  * that kernel leaves free (size it with max_ctas, e.g. the SM count minus
