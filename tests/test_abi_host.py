@@ -39,6 +39,27 @@ def test_exports_every_declared_symbol(tb):
     assert not missing, missing
 
 
+def _header_constants():
+    """NAME -> value of the header's integer #defines and enum members."""
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    consts = {}
+    for name, val in re.findall(r"^#define\s+(TB_[A-Z0-9_]+)\s+(.+?)\s*$", text, flags=re.M):
+        m = re.fullmatch(r"\(?\s*(\d+)u?\s*(?:<<\s*(\d+))?\s*\)?", val)
+        assert m, (name, val)
+        consts[name] = int(m.group(1)) << int(m.group(2) or 0)
+    for name, val in re.findall(r"\b(TB_[A-Z0-9_]+)\s*=\s*(\d+)", text):
+        consts[name] = int(val)
+    return consts
+
+
+def test_binding_constants_match_the_header(tb):
+    consts = _header_constants()
+    assert {"TB_OK", "TB_ERR_TIMEOUT", "TB_BF16", "TB_MAX_BATCH", "TB_EVICT_GATHER_CONCURRENT",
+            "TB_DECODE_CONCURRENT", "TB_NOALLOC_SCRATCH_BYTES"} <= set(consts)
+    for name, val in consts.items():
+        assert getattr(tb, name) == val, name
+
+
 def test_status_strings_and_version(tb):
     for s in range(6):
         assert tb.tb_status_string(s)
