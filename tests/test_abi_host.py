@@ -60,6 +60,35 @@ def test_binding_constants_match_the_header(tb):
         assert getattr(tb, name) == val, name
 
 
+def test_binding_structs_match_the_header(tb, tmp_path):
+    """Every field of the header's structs sits at the offset the ctypes
+    layout gives it, and the sizes agree (a C compiler reads the header)."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    pairs = [("tb_evict_desc", tb._EvictDescC), ("tb_decode_desc", tb._DecodeDescC),
+             ("tb_time_model", tb.TimeModel)]
+    lines = ["#include <stddef.h>", "#include <stdio.h>", '#include "timebill_kv.h"', "int main(void) {"]
+    for cname, py in pairs:
+        lines.append('  printf("%s sizeof %%zu\\n", sizeof(%s));' % (cname, cname))
+        for field, _ in py._fields_:
+            lines.append('  printf("%s %s %%zu\\n", offsetof(%s, %s));' % (cname, field, cname, field))
+    lines += ["  return 0;", "}"]
+    src, exe = tmp_path / "layout.c", tmp_path / "layout"
+    src.write_text("\n".join(lines) + "\n")
+    subprocess.run([cc, "-std=c11", "-I", os.path.dirname(HEADER), str(src), "-o", str(exe)], check=True)
+    got = {}
+    for line in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.splitlines():
+        cname, field, val = line.split()
+        got[(cname, field)] = int(val)
+    for cname, py in pairs:
+        assert got[(cname, "sizeof")] == ctypes.sizeof(py), cname
+        for field, _ in py._fields_:
+            assert got[(cname, field)] == getattr(py, field).offset, (cname, field)
+
+
 def test_status_strings_and_version(tb):
     for s in range(6):
         assert tb.tb_status_string(s)
