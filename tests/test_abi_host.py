@@ -89,6 +89,47 @@ def test_binding_structs_match_the_header(tb, tmp_path):
             assert got[(cname, field)] == getattr(py, field).offset, (cname, field)
 
 
+def _prototypes():
+    """name -> (return type, [parameter declarations]) of the header's functions."""
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    out = {}
+    for ret, name, args in re.findall(r"([A-Za-z_][\w \*]*?)\s*\b(tb_[a-z0-9_]+)\s*\(([^;{]*?)\)\s*;",
+                                      text, flags=re.S):
+        params = [a.strip() for a in args.replace("\n", " ").split(",")] if args.strip() not in ("", "void") else []
+        out[name] = (" ".join(ret.split()), params)
+    return out
+
+
+def _is_pointer_type(t):
+    return t in (ctypes.c_void_p, ctypes.c_char_p) or issubclass(t, ctypes._Pointer) or hasattr(t, "_dtype_")
+
+
+_SCALARS = {"int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64, "uint64_t": ctypes.c_uint64,
+            "size_t": ctypes.c_size_t, "double": ctypes.c_double, "tb_status": ctypes.c_int32}
+
+
+def test_binding_signatures_match_the_header(tb):
+    """Each entry point's ctypes argument list has the header's arity, a
+    pointer where the header has a pointer or a stream, and the header's
+    scalar type elsewhere; likewise the return type."""
+    protos = _prototypes()
+    assert set(protos) == set(_declared_functions())
+    lib = tb.load()
+    for name, (ret, params) in protos.items():
+        fn = getattr(lib, name)
+        assert fn.argtypes is not None and len(fn.argtypes) == len(params), name
+        for decl, t in zip(params, fn.argtypes):
+            if "*" in decl or decl.startswith("tb_stream_t"):
+                assert _is_pointer_type(t), (name, decl, t)
+            else:
+                ctype = decl.replace("const ", "").split()[0]
+                assert t is _SCALARS[ctype], (name, decl, t)
+        if "*" in ret:
+            assert fn.restype is ctypes.c_char_p, name
+        else:
+            assert fn.restype is _SCALARS[ret.split()[-1]], (name, ret)
+
+
 def test_status_strings_and_version(tb):
     for s in range(6):
         assert tb.tb_status_string(s)
