@@ -275,6 +275,15 @@ def profiled_traffic(stage, workload):
 STAGES = ["decode_attn", "window_scores", "select_topk", "gather_kv"]
 
 
+def pipelined_step(i, L):
+    """The C-ABI calls of step i of the pipelined layer loop over L >= 2
+    layer buffers, in stream order, as (call, buffer): layer i's scores and
+    select, then beside that select the decode over the cache compacted two
+    steps earlier and the gather of the rows selected one step earlier."""
+    return [("window_scores", i % L), ("select_topk", i % L),
+            ("decode_beside_select", (i + L - 2) % L), ("gather_beside_select", (i + L - 1) % L)]
+
+
 def to_device(torch, wl, x, dev):
     if wl.dtype == "bf16":
         return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
@@ -479,10 +488,8 @@ def run_ours(args, wl, alpha, world, rank, local, dist):
             for name in STAGES:
                 stage_call(name, d, cap)
         else:
-            stage_call("window_scores", d, cap)
-            stage_call("select_topk", d, cap)
-            stage_call("decode_beside_select", layers[(i + L - 2) % L], cap)
-            stage_call("gather_beside_select", layers[(i + L - 1) % L], cap)
+            for name, b in pipelined_step(i, L):
+                stage_call(name, layers[b], cap)
 
     step_graphs = []
     kernels_per_step = None
