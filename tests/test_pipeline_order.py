@@ -47,6 +47,16 @@ KERNELS = {
     "select_topk": [("select_cluster", True, "after_wait", False, ["scores"], ["idx", "ews"])],
     "decode_beside_select": [("decode_tma", False, "start", True, ["Kc", "sdws"], ["out", "sdws"])],
     "gather_beside_select": [("gather", False, "start", True, ["idx", "K", "V"], ["Kc"])],
+    # without the concurrent flag: the gather waits for the kernel before it
+    "gather_kv": [("gather", True, "after_wait", False, ["idx", "K", "V"], ["Kc"])],
+    # tb_score_evict: its clearing kernel, the scoring, the select, then its
+    # own gather (which never takes the concurrent flag)
+    "score_evict": [
+        ("clear_words", True, "after_wait", False, [], ["ews"]),
+        ("ws_tc", True, "exit", False, ["K", "q_win", "ews"], ["scores", "ews"]),
+        ("select_cluster", True, "after_wait", False, ["scores"], ["idx", "ews"]),
+        ("gather", True, "after_wait", False, ["idx", "K", "V"], ["Kc"]),
+    ],
 }
 
 
@@ -152,3 +162,23 @@ def test_the_schedule_touches_distinct_buffers_within_a_step():
             if L >= 3:
                 assert len({calls["window_scores"], calls["decode_beside_select"],
                             calls["gather_beside_select"]}) == 3
+
+
+@pytest.mark.parametrize("end_wait", [True, False])
+def test_the_gather_after_a_concurrent_decode_on_the_same_stream(end_wait):
+    """One layer's scores and select, the concurrent decode over another
+    layer's cache, then the plain gather of the select's rows on the same
+    stream (no event): the gather waits for the decode only, so its read of
+    the indices is ordered after the select exactly when the decode's grid
+    completes after the select."""
+    launch = [("window_scores", 0), ("select_topk", 0), ("decode_beside_select", 1), ("gather_kv", 0)]
+    ks, edges = _build([launch * 3], end_wait=end_wait)  # eager: one chain, no graph boundaries
+    bad = {(a, b, tuple(sh)) for a, b, _, sh in _unordered(ks, edges)}
+    assert bad == (set() if end_wait else {("select_cluster", "gather", ("idx",))})
+
+
+def test_score_evict_calls_in_a_row():
+    """tb_score_evict on one workspace and layer, call after call, eagerly
+    (every call its own launch sequence on one stream, PDL-chained)."""
+    ks, edges = _build([[("score_evict", 0)] * 4])
+    assert _unordered(ks, edges) == []
